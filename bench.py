@@ -1,0 +1,393 @@
+"""Benchmark of the per-chunk QuantWM KV-cache path on GB300.
+
+One step = one pass of the whole hot path for one new chunk of one layer:
+  attend   -- the chunk's queries attend over the packed history (every cached
+              chunk, with the PSAC logit term) and the active bf16 chunk;
+  append   -- the chunk's keys/values are QSAC-assigned, INT2-quantised,
+              PSAC-corrected and packed into a cache slot.
+Default workload: the Wan-14B-shaped layer (40 heads, head_dim 128, chunks of
+4680 tokens, 6 cached chunks = 28080 tokens, C=256, G=32, r=16, M=4).
+
+value  = attend FLOPs of the step / step time (whole-job, all ranks), TFLOP/s;
+the line also carries append GB/s and attend TFLOP/s with their roofline
+fractions, an end-to-end number through the public API with host buffers,
+the CPU oracle baseline and the SM clocks seen during the timed region.
+
+--impl reference times the CPU oracle (plain C, OpenMP over heads/rows) on a
+bounded sample of the same workload, scaled to the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "attend TFLOP/s + append GB/s per chunk, GB300 roofline % (1 GPU)"
+UNIT = "TFLOP/s"
+
+
+def workload_numbers(wl):
+    """Algorithmic work of one step (one layer-chunk)."""
+    H, d, N, C, G, r = wl.heads, wl.head_dim, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank
+    L = wl.cache_tokens
+    Nq = Ncur = N
+    attend_flops = 2.0 * H * Nq * (L * (2 * d + r) + Ncur * 2 * d)
+    ng = d // G
+    k_tok = d // 4 + 2 * ng + 1 + 1 + (r + 2 if r else 0)
+    v_tok = d // 4 + 2 * ng + 1 + 1
+    reads = 2 * N * H * d * 2 + 2 * H * C * d * 2 + H * d * r * 2 + H * d * 4
+    writes = N * H * (k_tok + v_tok) + 2 * H * C * d * 2 + H * r * d * 2
+    return {"attend_flops": attend_flops, "append_bytes": float(reads + writes),
+            "append_read_bytes": float(reads), "append_write_bytes": float(writes),
+            "k_bytes_per_token_head": k_tok, "v_bytes_per_token_head": v_tok}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"],
+                "bf16_tflops_sustained": j.get("bf16_tflops_sustained", j["bf16_tflops"]), "src": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="qwm_clocks_", suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, fl in rows for i, v in enumerate(fl) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------- GPU arm
+def run_gpu(args, wl, rank, world):
+    import torch
+    import paper_2609_26425_gb300 as qwm
+    from paper_2609_26425_gb300 import synth
+
+    local = int(os.environ.get("LOCAL_RANK", 0))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    qwm.lib()
+    H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, kmeans_iters=wl.kmeans_iters)
+    src = synth.ChunkSource(wl, layer=rank)
+    ws = torch.empty(qwm.qwm_fit_workspace_bytes(cfg, N), dtype=torch.uint8, device=dev)
+
+    def chunk_inputs(t):
+        q, k, v = src.chunk(t)
+        a = src.query_log_scale(t)
+        w = synth.population_w(a) if t > 0 else None
+        U = synth.population_U(a, r) if (t > 0 and r > 0) else None
+        return q, k, v, w, U
+
+    # history: past_chunks appended through the product path (centroids fitted on the GPU)
+    hist = qwm.Cache(cfg, N, wl.past_chunks, device=dev)
+    for t in range(wl.past_chunks):
+        _, k, v, w, U = chunk_inputs(t)
+        kd, vd = k.to(dev), v.to(dev)
+        kc = qwm.qwm_fit_centroids(cfg, kd, workspace=ws)
+        vc = qwm.qwm_fit_centroids(cfg, vd, workspace=ws)
+        qwm.qwm_quantize_append(cfg, hist, kd, vd, kc, vc, w=None if w is None else w.to(dev),
+                                U=None if U is None else U.to(dev))
+    # the new chunk
+    q, k, v, w, U = chunk_inputs(wl.past_chunks)
+    qd, kd, vd = q.to(dev), k.to(dev), v.to(dev)
+    wd = w.to(dev) if w is not None else None
+    Ud = U.to(dev) if U is not None else None
+    kc = qwm.qwm_fit_centroids(cfg, kd, workspace=ws)
+    vc = qwm.qwm_fit_centroids(cfg, vd, workspace=ws)
+    ring = qwm.Cache(cfg, N, 1, sliding_window=True, device=dev)  # the new chunk's slot
+    out = torch.empty_like(qd)
+    torch.cuda.synchronize()
+
+    nums = workload_numbers(wl)
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        qwm.qwm_attend(cfg, hist, qd, kd, vd, out=out)
+        if ev is not None:
+            ev[1].record(stream)
+        qwm.qwm_quantize_append(cfg, ring, kd, vd, kc, vc, w=wd, U=Ud)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    st = hist.status() | ring.status()
+    if st:
+        raise RuntimeError(f"device status {st} after the timed region")
+    ms = t0.elapsed_time(t1)
+    att_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
+    app_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+
+    # ---- end to end through the public API with host buffers
+    pin = lambda t: t.pin_memory()
+    hq, hk, hv = pin(q), pin(k), pin(v)
+    hkc, hvc = pin(kc.cpu()), pin(vc.cpu())
+    hw = pin(w) if w is not None else None
+    hU = pin(U) if U is not None else None
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
+    dkc, dvc = torch.empty_like(kc), torch.empty_like(vc)
+    dw = torch.empty_like(wd) if wd is not None else None
+    dU = torch.empty_like(Ud) if Ud is not None else None
+    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hkc, hvc) if t is not None)
+    h2d += sum(t.numel() * t.element_size() for t in (hw, hU) if t is not None)
+    d2h = hout.numel() * hout.element_size()
+
+    def e2e_step():
+        for h_, d_ in ((hq, dq), (hk, dk), (hv, dv), (hkc, dkc), (hvc, dvc), (hw, dw), (hU, dU)):
+            if h_ is not None:
+                d_.copy_(h_, non_blocking=True)
+        qwm.qwm_attend(cfg, hist, dq, dk, dv, out=out)
+        qwm.qwm_quantize_append(cfg, ring, dk, dv, dkc, dvc, w=dw, U=dU)
+        hout.copy_(out, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([e_ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        e_ms = float(tt.item())
+
+    pk = peaks()
+    att_tflops = nums["attend_flops"] / (att_ms * 1e-3) / 1e12
+    app_gbs = nums["append_bytes"] / (app_ms * 1e-3) / 1e9
+    value = world * args.steps * nums["attend_flops"] / (ms * 1e-3) / 1e12
+    e2e_value = world * args.steps * nums["attend_flops"] / (e_ms * 1e-3) / 1e12
+    res = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "heads": H, "head_dim": wl.head_dim, "chunk_tokens": N,
+                   "cached_tokens": wl.cache_tokens, "active_tokens": N, "query_tokens": N,
+                   "centroids": C, "group_size": G, "psac_rank": r, "candidates": M,
+                   "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (packed history %.0f MB + q/k/v %.0f MB per step)" % (
+                       hist.nbytes / 1e6, 3 * qd.numel() * 2 / 1e6)},
+        "attend": {"ms": round(att_ms, 4), "tflops": round(att_tflops, 2),
+                   "frac_of_measured_bf16": round(att_tflops / pk["bf16_tflops_sustained"], 4)},
+        "append": {"ms": round(app_ms, 4), "gbs": round(app_gbs, 1),
+                   "frac_of_measured_hbm": round(app_gbs / pk["hbm_gbs"], 4),
+                   "algorithmic_bytes": nums["append_bytes"]},
+        "roofline": {"bound": "tensor", "kernel": "attend_kernel", "achieved": round(att_tflops, 2),
+                     "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s",
+                     "frac": round(att_tflops / pk["bf16_tflops_sustained"], 4), "traffic": None,
+                     "peak_src": pk["src"] + " sustained bf16"},
+        "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk,
+    }
+    return res
+
+
+# ---------------------------------------------------------------------------- CPU oracle
+def oracle_sample(wl, append_tokens, attend_rows, attend_heads, nthreads):
+    """Time the CPU oracle on a bounded sample of one step and scale to a full step.
+    Returns (seconds per full step (extrapolated), description, cores)."""
+    import numpy as np
+    from oracle import oracle as orc
+    from paper_2609_26425_gb300 import synth
+
+    H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
+    src = synth.ChunkSource(wl)
+    q, k, v = src.chunk(wl.past_chunks)
+    kb, vb = synth.bits(k), synth.bits(v)
+    a = src.query_log_scale(wl.past_chunks)
+    w = synth.population_w(a).numpy()
+    Ub = synth.bits(synth.population_U(a, r))
+    idx = (np.arange(C) * N) // C
+    kc = np.ascontiguousarray(kb[idx].transpose(1, 0, 2))
+    vc = np.ascontiguousarray(vb[idx].transpose(1, 0, 2))
+    n_app = min(append_tokens, N)
+    t0 = time.perf_counter()
+    ko = orc.quantize(kb[:n_app], kc, G=G, r=r, M=M, is_key=True, w=w, U_bits=Ub, nthreads=nthreads)
+    vo = orc.quantize(vb[:n_app], vc, G=G, r=r, M=M, is_key=False, nthreads=nthreads)
+    t_app = time.perf_counter() - t0
+    # attention sample: attend_heads heads, attend_rows query rows, full key length
+    hs = list(range(attend_heads))
+    L = wl.cache_tokens + N
+    rng = np.random.default_rng(0)
+    Kf = rng.standard_normal((L, attend_heads, wl.head_dim))
+    Vf = rng.standard_normal((L, attend_heads, wl.head_dim))
+    # reconstruction cost of the sample's cached keys/values is part of the oracle's attend
+    t0 = time.perf_counter()
+    sub = {kk: vv[:, hs] for kk, vv in ko.items() if isinstance(vv, np.ndarray) and vv.ndim >= 2}
+    orc.dequant(sub, kc[hs], G=G, r=r, U_bits=Ub[hs])
+    t_deq_tok = (time.perf_counter() - t0) / n_app
+    rows = np.arange(attend_rows, dtype=np.int64)
+    t0 = time.perf_counter()
+    orc.attend(np.ascontiguousarray(synth.bits(q)[:, hs]), Kf, Vf, 1 / math.sqrt(wl.head_dim), rows=rows,
+               nthreads=nthreads)
+    t_att = time.perf_counter() - t0
+    full = (t_app * N / n_app
+            + t_deq_tok * 2 * wl.cache_tokens * H / attend_heads
+            + t_att * (N / attend_rows) * (H / attend_heads))
+    desc = (f"append: {n_app} of {N} tokens x {H} heads (K+V), scaled x{N / n_app:.1f}; attend: {attend_rows} "
+            f"query rows x {attend_heads} of {H} heads over all {L} keys, scaled x"
+            f"{(N / attend_rows) * (H / attend_heads):.0f}; reconstruction per token-head scaled to the cache")
+    return full, desc, (t_app + t_att)
+
+
+def cpu_baseline(wl, nthreads, append_tokens=512, attend_rows=32, attend_heads=4):
+    from oracle import oracle as orc
+    cores = nthreads if nthreads > 0 else orc.max_threads()
+    full, desc, spent = oracle_sample(wl, append_tokens, attend_rows, attend_heads, nthreads)
+    nums = workload_numbers(wl)
+    return {"value": round(nums["attend_flops"] / full / 1e12, 6), "unit": UNIT, "cores": cores,
+            "kind": "oracle", "sample": desc, "sample_seconds": round(spent, 2),
+            "seconds_per_step_extrapolated": round(full, 2)}
+
+
+def run_reference(args, wl):
+    from oracle import oracle as orc
+    orc.build()
+    nthreads = args.cpu_threads
+    cores = nthreads if nthreads > 0 else orc.max_threads()
+    for _ in range(args.warmup):
+        oracle_sample(wl, 64, 4, 2, nthreads)
+    times, desc = [], ""
+    for _ in range(args.steps):
+        full, desc, _ = oracle_sample(wl, 128, 8, 2, nthreads)
+        times.append(full)
+    nums = workload_numbers(wl)
+    sec = sum(times) / len(times)
+    value = nums["attend_flops"] / sec / 1e12
+    return {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "impl": "reference", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec * 1e3, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32/f64",
+            "data": "synthetic", "config": {"workload": wl.name, "heads": wl.heads, "chunk_tokens": wl.chunk_tokens,
+                                            "cached_tokens": wl.cache_tokens},
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="qwm", choices=["qwm", "reference"])
+    ap.add_argument("--workload", default="wan14b_layer")
+    ap.add_argument("--cpu-threads", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    from paper_2609_26425_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args, wl)), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        torch.distributed.init_process_group("nccl")
+    res = run_gpu(args, wl, rank, world)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        if not args.no_cpu_baseline and world == 1:
+            res["cpu_baseline"] = cpu_baseline(wl, args.cpu_threads)
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

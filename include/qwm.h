@@ -1,0 +1,175 @@
+/*
+ * qwm.h -- C ABI of the GB300-native QuantWM per-chunk 2-bit KV-cache path.
+ *
+ * QuantWM ("Temporally Consistent 2-Bit KV Cache Quantization for Video World
+ * Models") stores each finished chunk of an autoregressive video model's KV
+ * cache as centroid ids + INT2 residual codes (Sec. 2 Eq. 1-4), chosen by the
+ * Query-sensitivity-aware QSAC rule (Sec. 4.1 Eq. 9-12), plus for Keys a
+ * rank-r PSAC correction C = E U_r (Sec. 4.2 Eq. 13-17); attention then runs
+ * over the packed history and the active bf16 chunk (App. D.1 "Cache
+ * lifecycle").  This library implements both halves of that per-chunk path on
+ * one GB300 GPU (sm_103a):
+ *   qwm_fit_centroids    k-means centroids of a chunk (Sec. 2, QVG convention)
+ *   qwm_quantize_append  QSAC assignment, INT2 residual quantization + packing,
+ *                        PSAC coefficients, written into one chunk slot
+ *   qwm_attend           softmax attention of new queries over the packed
+ *                        chunks (with the PSAC logit term Q U_r C^T) and the
+ *                        active bf16 chunk
+ *   qwm_cache_bytes      size of the caller-owned cache buffer
+ *
+ * Conventions for every call:
+ *   - Tensor pointers are DEVICE pointers owned by the caller; the library
+ *     never allocates device memory.  bf16 tensors are token-major
+ *     [tokens][heads][head_dim], contiguous, 16-byte aligned.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream); every call is
+ *     asynchronous on it, except qwm_cache_status, which synchronises it.
+ *   - Host-detectable errors (bad arguments, unsupported shapes, capacity)
+ *     are returned before anything is launched.  Errors detected on the GPU
+ *     (a bounded wait that ran out) are recorded in the cache's device status
+ *     word, read with qwm_cache_status.
+ *   - Supported: head_dim 128; group_size 32 or 64; 1 <= num_centroids <= 256;
+ *     psac_rank 0, 8, 16 or 32; num_candidates >= 1 (values above
+ *     num_centroids mean "all centroids").  Anything else returns
+ *     QWM_ERR_UNSUPPORTED.
+ */
+#ifndef QWM_H
+#define QWM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define QWM_API __attribute__((visibility("default")))
+#else
+#define QWM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Problem statement: heads H, head_dim d, centroid count C, INT2 group size G,
+ * PSAC rank r (Sec. 4.2; r = 0 disables PSAC), QSAC candidate count M
+ * (App. C.5, default 4), Lloyd iterations of qwm_fit_centroids. */
+typedef struct qwm_config {
+  int32_t num_heads;
+  int32_t head_dim;
+  int32_t num_centroids;
+  int32_t group_size;
+  int32_t psac_rank;
+  int32_t num_candidates;
+  int32_t kmeans_iters;
+} qwm_config;
+
+typedef enum qwm_status {
+  QWM_OK = 0,
+  QWM_ERR_INVALID_ARG = 1, /* NULL pointer, negative size, mismatched config */
+  QWM_ERR_UNSUPPORTED = 2, /* shape outside the supported set above */
+  QWM_ERR_CAPACITY = 3,    /* chunk larger than a slot, or cache full without a window */
+  QWM_ERR_CUDA = 4,        /* a CUDA runtime call failed */
+  QWM_ERR_TIMEOUT = 5,     /* a bounded wait inside a kernel ran out (device status) */
+  QWM_ERR_NONFINITE = 6    /* reserved for non-finite inputs */
+} qwm_status;
+
+/* Opaque host descriptor over a caller-owned device buffer. */
+typedef struct qwm_cache qwm_cache;
+
+/* Byte offsets of the packed cache, for readers of the buffer (tests, tools).
+ * A slot holds one chunk: for head h, at slot_offset(s) + slot_meta_bytes +
+ * h*head_bytes, come the Key centroid table [C][d] bf16, the Value centroid
+ * table [C][d] bf16, U_r^T [r][d] bf16, then tiles_per_chunk tiles of
+ * tile_tokens tokens.  Each tile is a Key block followed by a Value block of
+ * structure-of-arrays fields (offsets within the tile): codes [128][d/4] u8
+ * (channel c in byte c/4, bits 2(c%4)), scales [128][d/G] binary16,
+ * ids [128] u8, zero-points [128][zb] u8 (group g in byte g/4, bits 2(g%4)),
+ * and for Keys PSAC codes [128][r] int8 and row scales [128] binary16. */
+typedef struct qwm_layout {
+  int64_t header_bytes;     /* device status word + reserved, before slot 0 */
+  int64_t slot_meta_bytes;  /* per-slot reserved bytes before head 0 */
+  int64_t slot_bytes;       /* bytes per chunk slot */
+  int64_t head_bytes;       /* bytes per head inside a slot */
+  int64_t ktab_offset, vtab_offset, ut_offset, tiles_offset; /* within a head */
+  int64_t tile_tokens, tiles_per_chunk, tile_bytes;
+  int64_t k_codes, k_scales, k_ids, k_zeros, k_coef, k_sigma, k_bytes; /* within a tile */
+  int64_t v_codes, v_scales, v_ids, v_zeros, v_bytes; /* within a tile, from its start */
+  int64_t zero_bytes;       /* zb: bytes of packed zero-points per token */
+} qwm_layout;
+
+/* Human-readable name of a status code (static string). */
+QWM_API const char* qwm_status_string(qwm_status status);
+
+/* Bytes of device memory a cache of max_chunks slots of tokens_per_chunk
+ * tokens needs (App. D.1 packed storage: per token-head d/4 code bytes, d/G
+ * binary16 scales, one uint8 centroid id, 2-bit zero-points, for Keys r INT8
+ * PSAC codes + one binary16 row scale; per chunk-head the two bf16 centroid
+ * tables and U_r).  Returns 0 for an invalid or unsupported configuration. */
+QWM_API size_t qwm_cache_bytes(const qwm_config* cfg, int64_t tokens_per_chunk, int32_t max_chunks);
+
+/* Create a host descriptor over dev_buf (256-byte aligned, bytes >=
+ * qwm_cache_bytes(...)), and
+ * clear the buffer's header on `stream`.  max_chunks <= 256.  With
+ * sliding_window != 0, appending to a full cache overwrites the oldest chunk
+ * (slot = chunk index mod max_chunks); otherwise it returns QWM_ERR_CAPACITY.
+ * The descriptor is freed with qwm_cache_free; the buffer stays the caller's. */
+QWM_API qwm_status qwm_cache_init(qwm_cache** out, const qwm_config* cfg, void* dev_buf, size_t bytes,
+                          int64_t tokens_per_chunk, int32_t max_chunks, int32_t sliding_window,
+                          void* stream);
+QWM_API void qwm_cache_free(qwm_cache* cache);
+
+/* Number of chunks currently held; chunk i (0 = oldest) lives in *slot and
+ * has *tokens tokens. */
+QWM_API int32_t qwm_cache_num_chunks(const qwm_cache* cache);
+QWM_API qwm_status qwm_cache_chunk_info(const qwm_cache* cache, int32_t i, int32_t* slot, int64_t* tokens);
+QWM_API qwm_status qwm_cache_layout(const qwm_cache* cache, qwm_layout* out);
+
+/* Synchronise `stream`, then read and clear the device status word: *status
+ * receives QWM_OK or the first error a kernel recorded (QWM_ERR_TIMEOUT). */
+QWM_API qwm_status qwm_cache_status(qwm_cache* cache, int32_t* status, void* stream);
+
+/* Scratch bytes qwm_fit_centroids needs for N tokens (fp32 centroids, fp64
+ * member sums and counts); 0 for an invalid configuration. */
+QWM_API size_t qwm_fit_workspace_bytes(const qwm_config* cfg, int64_t N);
+
+/* k-means centroids of one chunk, per head (Sec. 2: centroid-residual form of
+ * QVG, fitted with Lloyd's algorithm; App. D.1 keeps centroids in BF16).
+ * x: bf16 [N][H][d] (N >= 1).  centroids (out): bf16 [H][C][d].
+ * Initial centroid j is token floor(j*N/C); each of kmeans_iters iterations
+ * assigns every token to its Euclidean-nearest centroid (ties to the lower
+ * index) and replaces each non-empty cluster's centroid by its member mean;
+ * the result is rounded to bf16.  workspace: device scratch of at least
+ * qwm_fit_workspace_bytes(cfg, N) bytes, 256-byte aligned. */
+QWM_API qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, void* centroids,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Quantize one finished chunk and append it to the cache (Sec. 4.1 QSAC,
+ * Sec. 2 Eq. 1-4 INT2 residuals, Sec. 4.2 Eq. 13/16 PSAC, App. D.1 packing).
+ * k, v: bf16 [N][H][d], 1 <= N <= tokens_per_chunk.  k_centroids,
+ * v_centroids: bf16 [H][C][d] (this chunk's tables; copied into the slot).
+ * w: fp32 [H][d] channel sensitivity weights (Eq. 8) or NULL for w = 1 (the
+ * cold-start rule of App. C.3).  U: bf16 [H][d][r] principal Query basis
+ * (Eq. 15) or NULL to store no PSAC correction (cold start).  Keys: top-M
+ * candidates by the Query-aware distance (Eq. 9), then the lowest QSAC score
+ * (Eq. 12), ties to the lower index; Values: the same with w = 1 and no PSAC.
+ * The chunk goes to the next slot (oldest slot when a sliding window is full). */
+QWM_API qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* cache, const void* k, const void* v,
+                               int64_t N, const void* k_centroids, const void* v_centroids,
+                               const float* w, const void* U, void* stream);
+
+/* Attention of Nq new queries over every cached chunk and the active chunk
+ * (Sec. 3.3 Eq. 5 logits; Sec. 4.2 Eq. 17: Q K_hat^T = Q K_hat0^T +
+ * (Q U_r) C^T with each chunk's own U_r; Values rebuilt without PSAC).
+ * q: bf16 [Nq][H][d]; k_cur, v_cur: bf16 [N_cur][H][d] of the active chunk
+ * (N_cur = 0 allowed, then they may be NULL).  No mask: cached chunks are in
+ * the past.  sm_scale > 0 (usually 1/sqrt(d)).
+ * out: bf16 [Nq][H][d] = softmax(sm_scale * logits) V.
+ * lse: fp32 [H][Nq] natural-log sum-exp of the scaled logits, or NULL.
+ * At least one key (a cached chunk or N_cur > 0) is required. */
+QWM_API qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* cache, const void* q, int64_t Nq,
+                      const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,
+                      void* out, float* lse, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QWM_H */

@@ -1,0 +1,125 @@
+// qwm_internal.cuh -- shared definitions of the CUDA library: cache layout,
+// kernel parameter blocks, launch entry points and sm_103a PTX helpers
+// (tcgen05, mbarrier, bulk copies).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "../../include/qwm.h"
+
+namespace qwm {
+
+constexpr int kHeadDim = 128;
+constexpr int kTile = 128;        // tokens per cache tile, queries per attend CTA
+constexpr int kMaxSlots = 256;    // chunk slots per cache
+constexpr int kHeaderBytes = 256;
+constexpr int kSlotMetaBytes = 256;
+
+__host__ __device__ inline int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+// Byte layout of the packed cache (see qwm_layout in qwm.h).
+struct Layout {
+  int H, d, C, G, r, ng, zb;
+  int64_t T;             // token capacity of a slot
+  int32_t max_chunks;
+  int64_t tiles;         // tiles per slot
+  int64_t k_codes, k_scales, k_ids, k_zeros, k_coef, k_sigma, k_bytes;
+  int64_t v_codes, v_scales, v_ids, v_zeros, v_bytes;  // from the tile start
+  int64_t tile_bytes;
+  int64_t ktab, vtab, ut, tiles_off, head_bytes;
+  int64_t slot_bytes;
+  int64_t total_bytes;
+};
+
+inline Layout make_layout(const qwm_config& c, int64_t T, int32_t max_chunks) {
+  Layout L{};
+  L.H = c.num_heads; L.d = c.head_dim; L.C = c.num_centroids; L.G = c.group_size; L.r = c.psac_rank;
+  L.ng = L.d / L.G;
+  L.zb = (2 * L.ng + 7) / 8;
+  L.T = T; L.max_chunks = max_chunks;
+  L.tiles = (T + kTile - 1) / kTile;
+  int64_t o = 0;
+  L.k_codes = o;  o += (int64_t)kTile * (L.d / 4);
+  L.k_scales = o; o += round_up((int64_t)kTile * L.ng * 2, 16);
+  L.k_ids = o;    o += kTile;
+  L.k_zeros = o;  o += round_up((int64_t)kTile * L.zb, 16);
+  L.k_coef = o;   o += (int64_t)kTile * L.r;
+  L.k_sigma = o;  o += L.r > 0 ? kTile * 2 : 0;
+  L.k_bytes = round_up(o, 128);
+  o = L.k_bytes;
+  L.v_codes = o;  o += (int64_t)kTile * (L.d / 4);
+  L.v_scales = o; o += round_up((int64_t)kTile * L.ng * 2, 16);
+  L.v_ids = o;    o += kTile;
+  L.v_zeros = o;  o += round_up((int64_t)kTile * L.zb, 16);
+  L.v_bytes = round_up(o, 128) - L.k_bytes;
+  L.tile_bytes = L.k_bytes + L.v_bytes;
+  o = 0;
+  L.ktab = o;      o += (int64_t)L.C * L.d * 2;
+  L.vtab = o;      o += (int64_t)L.C * L.d * 2;
+  L.ut = o;        o += (int64_t)L.r * L.d * 2;
+  o = round_up(o, 1024);
+  L.tiles_off = o; o += L.tiles * L.tile_bytes;
+  L.head_bytes = round_up(o, 1024);
+  L.slot_bytes = kSlotMetaBytes + (int64_t)L.H * L.head_bytes;
+  L.total_bytes = kHeaderBytes + (int64_t)max_chunks * L.slot_bytes;
+  return L;
+}
+
+__host__ __device__ inline int64_t head_offset(const Layout& L, int slot, int h) {
+  return kHeaderBytes + (int64_t)slot * L.slot_bytes + kSlotMetaBytes + (int64_t)h * L.head_bytes;
+}
+
+// ----------------------------------------------------------------------------
+// Kernel launch entry points (defined in the .cu files).
+// ----------------------------------------------------------------------------
+struct AppendArgs {
+  Layout L;
+  uint8_t* base;               // cache buffer
+  int slot;
+  int64_t N;
+  const __nv_bfloat16* k;      // [N][H][d]
+  const __nv_bfloat16* v;
+  const __nv_bfloat16* kc;     // [H][C][d]
+  const __nv_bfloat16* vc;
+  const float* w;              // [H][d] or null
+  const __nv_bfloat16* U;      // [H][d][r] or null
+  int M;                       // candidates (clamped to C)
+};
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
+
+struct AttendSlots {
+  int32_t n;
+  int32_t slot[kMaxSlots];
+  int32_t tokens[kMaxSlots];
+  int32_t psac[kMaxSlots];     // chunk stored with a PSAC correction
+};
+struct AttendArgs {
+  Layout L;
+  const uint8_t* base;
+  int32_t* status;             // device status word
+  const __nv_bfloat16* q;      // [Nq][H][d]
+  const __nv_bfloat16* kcur;   // [Ncur][H][d]
+  const __nv_bfloat16* vcur;
+  int64_t Nq, Ncur;
+  float sm_scale;
+  __nv_bfloat16* out;          // [Nq][H][d]
+  float* lse;                  // [H][Nq] or null
+};
+cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t s);
+
+struct FitArgs {
+  int H, d, C, iters;
+  int64_t N;
+  const __nv_bfloat16* x;      // [N][H][d]
+  __nv_bfloat16* out;          // [H][C][d]
+  float* cent;                 // workspace: [H][C][d] fp32
+  double* sums;                // workspace: [H][C][d] fp64
+  uint32_t* counts;            // workspace: [H][C]
+};
+size_t fit_workspace_bytes(int H, int d, int C);
+cudaError_t launch_fit(const FitArgs& a, cudaStream_t s);
+
+}  // namespace qwm

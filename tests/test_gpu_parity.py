@@ -1,0 +1,241 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Inputs are seeded synthetic tensors from paper_2609_26425_gb300.synth; the
+centroid tables fed to both sides come from the oracle's k-means or from the
+generator, never from the GPU.  Packed codes, zero-points, scales and ids are
+compared bit-exactly (with the oracle-margin rule for near-ties), attention
+against the oracle's fp64 softmax attention over the oracle's own
+reconstruction.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2609_26425_gb300 import synth
+import paper_2609_26425_gb300 as qwm
+
+from parity import compare_attention, compare_packed, oracle_append, oracle_kv
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    qwm.lib()
+
+
+def dev(t):
+    return t.to("cuda").contiguous()
+
+
+def strided_centroids(x_bits, C):
+    """Generator-side centroid table: tokens floor(j*N/C) of the chunk (no arithmetic)."""
+    N = x_bits.shape[0]
+    idx = (np.arange(C) * N) // C
+    return np.ascontiguousarray(x_bits[idx].transpose(1, 0, 2))
+
+
+def make_chunk(seed, N, H, *, outliers=True):
+    q = synth.gaussian_bf16(seed * 3 + 1, N, H, 128)
+    k = synth.gaussian_bf16(seed * 3 + 2, N, H, 128)
+    if outliers:
+        k = k.float()
+        k[:, :, [5, 40, 77, 120]] *= 8
+        k = k.to(torch.bfloat16)
+    v = synth.gaussian_bf16(seed * 3 + 3, N, H, 128)
+    return q, k, v
+
+
+def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None):
+    _, k, v = make_chunk(seed, N, H)
+    kb, vb = synth.bits(k), synth.bits(v)
+    if fit_iters:
+        kc = orc.fit_centroids(kb, C, fit_iters)["centroids"]
+        vc = orc.fit_centroids(vb, C, fit_iters)["centroids"]
+    else:
+        kc, vc = strided_centroids(kb, C), strided_centroids(vb, C)
+    w = synth.random_weights(seed + 100, H, 128).numpy() if use_w else None
+    Ub = synth.bits(synth.random_orthonormal(seed + 200, H, 128, r)) if (use_U and r > 0) else None
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    cache = qwm.Cache(cfg, T or N, 2)
+    qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
+                            w=None if w is None else torch.from_numpy(w).cuda(),
+                            U=None if Ub is None else dev(synth.from_bits(Ub)))
+    torch.cuda.synchronize()
+    assert cache.status() == 0
+    dec = cache.decode_chunk(0)
+    ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub)
+    sk = compare_packed(dec, ko, kb, kc, G=G, r=r, M=M, is_key=True, w=w, U_bits=Ub)
+    sv = compare_packed(dec, vo, vb, vc, G=G, r=r, M=M, is_key=False, prefix="v_")
+    assert np.array_equal(dec["k_tab"], kc) and np.array_equal(dec["v_tab"], vc)
+    if Ub is not None:
+        assert np.array_equal(dec["U"], Ub)
+    return sk, sv
+
+
+@pytest.mark.parametrize("H,N,C,G,r,M,use_w,use_U", [
+    (4, 880, 64, 32, 16, 4, True, True),      # the single-layer workload's shape
+    (2, 300, 16, 64, 8, 4, True, True),
+    (2, 257, 256, 32, 32, 4, True, True),
+    (3, 130, 64, 32, 16, 1, False, False),    # cold start: w = 1, no PSAC
+    (2, 200, 8, 32, 16, 8, True, True),       # exhaustive QSAC (M = C)
+    (2, 129, 64, 64, 0, 4, True, False),      # PSAC disabled by rank 0
+    (1, 1, 4, 32, 8, 4, True, True),          # a single token
+])
+def test_append_parity(H, N, C, G, r, M, use_w, use_U):
+    sk, sv = run_append_case(H, N, C, G, r, M, use_w, use_U, seed=H * 1000 + N)
+    assert sk["id_flips"] <= max(1, N * H // 1000)
+
+
+def test_append_parity_fitted_tables():
+    """Tables from the oracle's k-means (the realistic case: many near ties)."""
+    run_append_case(4, 880, 64, 32, 16, 4, True, True, seed=7, fit_iters=10)
+
+
+def test_fit_parity():
+    H, N, C, iters = 4, 880, 64, 10
+    _, k, _ = make_chunk(11, N, H)
+    kb = synth.bits(k)
+    ref = orc.fit_centroids(kb, C, iters)
+    cfg = qwm.config(H, C, kmeans_iters=iters)
+    got = qwm.qwm_fit_centroids(cfg, dev(k))
+    torch.cuda.synchronize()
+    g = synth.bits(got.cpu())
+    # same assignments against both tables, and the k-means objective agrees
+    exact = np.array_equal(g, ref["centroids"])
+    xf = orc.bf16_to_f32(kb).astype(np.float64)
+    for h in range(H):
+        cg = orc.bf16_to_f32(g[h]).astype(np.float64)
+        cr = orc.bf16_to_f32(ref["centroids"][h]).astype(np.float64)
+        dg = ((xf[:, h, None, :] - cg[None]) ** 2).sum(-1)
+        dr = ((xf[:, h, None, :] - cr[None]) ** 2).sum(-1)
+        agree = (dg.argmin(1) == dr.argmin(1)).mean()
+        assert agree >= 0.999 or exact
+        og, orf = dg.min(1).sum(), dr.min(1).sum()
+        assert abs(og - orf) <= 1e-4 * orf
+    # k = C = 1 iteration-free case: init tokens exactly
+    cfg0 = qwm.config(H, C, kmeans_iters=0)
+    got0 = synth.bits(qwm.qwm_fit_centroids(cfg0, dev(k)).cpu())
+    assert np.array_equal(got0, orc.fit_centroids(kb, C, 0)["centroids"])
+
+
+def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, window=0, max_chunks=None,
+                              psac_chunks=None, rows=None):
+    """Append chunks on the GPU and build the oracle's reference keys/values."""
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    T = max(chunk_sizes)
+    cache = qwm.Cache(cfg, T, max_chunks or len(chunk_sizes), sliding_window=bool(window))
+    Ks, Vs = [], []
+    for ci, N in enumerate(chunk_sizes):
+        _, k, v = make_chunk(seed + ci, N, H)
+        kb, vb = synth.bits(k), synth.bits(v)
+        kc, vc = strided_centroids(kb, C), strided_centroids(vb, C)
+        use_psac = r > 0 and (psac_chunks is None or ci in psac_chunks)
+        w = synth.random_weights(seed + 50 + ci, H, 128).numpy() if ci > 0 else None
+        Ub = synth.bits(synth.random_orthonormal(seed + 80 + ci, H, 128, r)) if use_psac else None
+        qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
+                                w=None if w is None else torch.from_numpy(w).cuda(),
+                                U=None if Ub is None else dev(synth.from_bits(Ub)))
+        ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub)
+        K, V = oracle_kv(ko, vo, kc, vc, G=G, r=r, U_bits=Ub)
+        Ks.append(K)
+        Vs.append(V)
+    n_keep = cache.num_chunks
+    Ks, Vs = Ks[len(Ks) - n_keep:], Vs[len(Vs) - n_keep:]
+    q, kcur, vcur = make_chunk(seed + 999, max(Nq, Ncur, 1), H, outliers=True)
+    q = q[:Nq].contiguous()
+    kcur, vcur = kcur[:Ncur].contiguous(), vcur[:Ncur].contiguous()
+    if Ncur:
+        Ks.append(orc.bf16_to_f32(synth.bits(kcur)).astype(np.float64))
+        Vs.append(orc.bf16_to_f32(synth.bits(vcur)).astype(np.float64))
+    Kall, Vall = np.concatenate(Ks, 0), np.concatenate(Vs, 0)
+    scale = 1 / math.sqrt(128)
+    ref, lse = orc.attend(synth.bits(q), Kall, Vall, scale, rows=rows)
+    return cfg, cache, q, kcur, vcur, ref, lse
+
+
+@pytest.mark.parametrize("H,chunks,C,G,r,Ncur,Nq", [
+    (4, [880, 880], 64, 32, 16, 880, 880),    # the single-layer workload
+    (2, [300, 77], 16, 64, 8, 129, 200),
+    (2, [256, 256], 256, 32, 32, 0, 130),     # no active chunk
+    (2, [128], 64, 32, 0, 1, 1),              # r = 0, one query, one active key
+    (1, [1, 5], 4, 32, 16, 0, 33),            # tiny chunks
+])
+def test_attend_parity(H, chunks, C, G, r, Ncur, Nq):
+    cfg, cache, q, kc, vc, ref, lse = build_cache_and_reference(H, chunks, C, G, r, 4, seed=31 * H + Nq,
+                                                               Ncur=Ncur, Nq=Nq)
+    out, lse_g = qwm.qwm_attend(cfg, cache, dev(q), dev(kc) if Ncur else None, dev(vc) if Ncur else None,
+                                want_lse=True)
+    torch.cuda.synchronize()
+    assert cache.status() == 0
+    compare_attention(out.float().cpu().numpy(), ref)
+    assert np.abs(lse_g.cpu().numpy() - lse).max() < 2e-2
+
+
+def test_attend_sliding_window_and_cold_chunk():
+    """A ring of 2 slots after 4 appends holds the last two chunks; the first
+    held chunk was appended without PSAC (cold start)."""
+    cfg, cache, q, kc, vc, ref, _ = build_cache_and_reference(2, [200, 150, 180, 90], 16, 32, 16, 4, seed=5,
+                                                             Ncur=64, Nq=100, window=1, max_chunks=2,
+                                                             psac_chunks={3})
+    assert cache.num_chunks == 2
+    out = qwm.qwm_attend(cfg, cache, dev(q), dev(kc), dev(vc))
+    torch.cuda.synchronize()
+    compare_attention(out.float().cpu().numpy(), ref)
+
+
+def test_attend_lossless_cache_equals_dense_attention():
+    """Keys/values on the INT2 grid with a zero centroid reconstruct exactly, so
+    attention over the cache equals attention over the raw bf16 tensors."""
+    H, N, d, G = 2, 256, 128, 32
+    rng = np.random.default_rng(9)
+    s = 0.25
+    def grid():
+        m = rng.integers(-1, 3, size=(N, H, d)).astype(np.float32)
+        m[..., ::G] = -1
+        m[..., 1::G] = 2
+        return torch.from_numpy(m * s).to(torch.bfloat16)
+    k, v = grid(), grid()
+    q = synth.gaussian_bf16(10, 77, H, d)
+    cfg = qwm.config(H, 1, group_size=G, psac_rank=0, candidates=1)
+    cache = qwm.Cache(cfg, N, 1)
+    zc = torch.zeros(H, 1, d, dtype=torch.bfloat16)
+    qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(zc), dev(zc))
+    out = qwm.qwm_attend(cfg, cache, dev(q))
+    torch.cuda.synchronize()
+    qf = q.double().permute(1, 0, 2)
+    ref = torch.nn.functional.scaled_dot_product_attention(qf, k.double().permute(1, 0, 2),
+                                                           v.double().permute(1, 0, 2)).permute(1, 0, 2)
+    compare_attention(out.float().cpu().numpy(), ref.numpy())
+
+
+def test_error_paths():
+    H = 2
+    cfg = qwm.config(H, 16, group_size=32, psac_rank=16)
+    cache = qwm.Cache(cfg, 100, 1)
+    _, k, v = make_chunk(3, 101, H)
+    kc = dev(torch.zeros(H, 16, 128, dtype=torch.bfloat16))
+    with pytest.raises(qwm.QwmError) as e:
+        qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), kc, kc)
+    assert e.value.status == 3  # capacity
+    qwm.qwm_quantize_append(cfg, cache, dev(k[:100]), dev(v[:100]), kc, kc)
+    with pytest.raises(qwm.QwmError) as e:  # full, no sliding window
+        qwm.qwm_quantize_append(cfg, cache, dev(k[:10]), dev(v[:10]), kc, kc)
+    assert e.value.status == 3
+    bad = qwm.config(H, 16, group_size=16)
+    assert qwm.qwm_cache_bytes(bad, 100, 1) == 0
+    with pytest.raises(qwm.QwmError):
+        qwm.qwm_attend(cfg, cache, dev(k[:4]), sm_scale=-1.0)
+    empty = qwm.Cache(cfg, 100, 1)
+    with pytest.raises(qwm.QwmError) as e:  # no keys at all
+        qwm.qwm_attend(cfg, empty, dev(k[:4]))
+    assert e.value.status == 1
+    out = qwm.qwm_attend(cfg, cache, dev(k[:0]))  # Nq = 0 is a no-op
+    assert out.shape[0] == 0
+    torch.cuda.synchronize()
+    assert cache.status() == 0
