@@ -163,6 +163,9 @@ QWM_API qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* cache, 
  * the past.  sm_scale > 0 (usually 1/sqrt(d)).
  * out: bf16 [Nq][H][d] = softmax(sm_scale * logits) V.
  * lse: fp32 [H][Nq] natural-log sum-exp of the scaled logits, or NULL.
+ * The tensor-core operands are binary16 with fp32 accumulation, so q, k_cur,
+ * v_cur and the rebuilt cache values must lie within the binary16 range
+ * (|x| < 65504).
  * At least one key (a cached chunk or N_cur > 0) is required. */
 QWM_API qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* cache, const void* q, int64_t Nq,
                       const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,

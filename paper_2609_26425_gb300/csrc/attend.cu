@@ -3,8 +3,8 @@
 //
 // Per CTA: 128 queries of one head.  For every 128-key tile of every cached
 // chunk the CTA
-//   1. rebuilds K_hat0 = mu_id + s (q - z) (Sec. 2 Eq. 4) in shared memory as a
-//      bf16 MMA operand (128-byte swizzled, K-major), plus r extra columns
+//   1. rebuilds K_hat0 = mu_id + s (q - z) (Sec. 2 Eq. 4) in shared memory as an
+//      f16 MMA operand (128-byte swizzled, K-major), plus r extra columns
 //      C_hat = t * sigma of the PSAC coefficients (Sec. 4.2 Eq. 16),
 //   2. issues S = [Q | Q U_r] [K_hat0 | C_hat]^T on tcgen05 into TMEM: the
 //      PSAC logit correction Q U_r C^T (Eq. 17) rides along as r extra
@@ -16,7 +16,10 @@
 //      than 2^8, which keeps every P <= 2^8), writes P as bf16 operand,
 //   5. issues O += P V_hat on tcgen05 into TMEM.
 // The active chunk's dense bf16 K/V tiles run through the same loop without
-// the PSAC columns.  All mbarrier waits are bounded; a wait that runs out
+// the PSAC columns.  MMA operands are binary16 (11 significant bits; the
+// bf16 inputs convert exactly) with fp32 accumulation: same tensor rate as
+// bf16, but 8x finer rounding of the rebuilt keys, which keeps the logits of
+// outlier channels accurate.  Inputs must stay inside the binary16 range.  All mbarrier waits are bounded; a wait that runs out
 // records QWM_ERR_TIMEOUT in the cache's status word and the CTA leaves.
 #include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
@@ -80,7 +83,7 @@ __device__ __forceinline__ void dequant_row(uint8_t* dst, int row, const uint8_t
       const float q0 = (float)((bits >> (4 * p)) & 3u), q1 = (float)((bits >> (4 * p + 2)) & 3u);
       const float v0 = __uint_as_float(mw[p] << 16) + (q0 - zf) * s;
       const float v1 = __uint_as_float(mw[p] & 0xFFFF0000u) + (q1 - zf) * s;
-      ow[p] = pack_bf16(v0, v1);
+      ow[p] = pack_f16(v0, v1);
     }
     st_chunk(dst, row, ch, make_uint4(ow[0], ow[1], ow[2], ow[3]));
   }
@@ -92,7 +95,7 @@ __device__ __forceinline__ void zero_row(uint8_t* dst, int row, int nch) {
 
 __device__ __forceinline__ void copy_row(uint8_t* dst, int row, const __nv_bfloat16* src) {
 #pragma unroll
-  for (int ch = 0; ch < 16; ++ch) st_chunk(dst, row, ch, ldg16(src + ch * 8));
+  for (int ch = 0; ch < 16; ++ch) st_chunk(dst, row, ch, bf16x8_to_f16x8(ldg16(src + ch * 8)));
 }
 
 __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const AttendSlots S) {
@@ -138,8 +141,8 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
   if (r > 0) zero_row(sQ + 2 * BLK, tid, rpad / 8);
 
   const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV), aP = smem_u32(sP);
-  constexpr uint32_t idS = idesc_bf16(128, 128, false);
-  constexpr uint32_t idPV = idesc_bf16(128, 64, true);
+  constexpr uint32_t idS = idesc_f16(128, 128, false);
+  constexpr uint32_t idPV = idesc_f16(128, 64, true);
   const float sl2 = a.sm_scale * 1.4426950408889634f;
 
   float m_run = -INFINITY, l_run = 0.0f;
@@ -183,7 +186,7 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
 #pragma unroll
         for (int p = 0; p < 4; ++p) {
           const int j = c2 * 8 + 2 * p;
-          w4[p] = pack_bf16(j < r ? acc[j] : 0.0f, j + 1 < r ? acc[j + 1] : 0.0f);
+          w4[p] = pack_f16(j < r ? acc[j] : 0.0f, j + 1 < r ? acc[j + 1] : 0.0f);
         }
         st_chunk(sQ + 2 * BLK, tid, c2, make_uint4(w4[0], w4[1], w4[2], w4[3]));
       }
@@ -212,7 +215,7 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
                 const int j = c2 * 8 + 2 * p;
                 const float t0 = j < r ? (float)cp[j] * sg : 0.0f;
                 const float t1 = j + 1 < r ? (float)cp[j + 1] * sg : 0.0f;
-                w4[p] = pack_bf16(t0, t1);
+                w4[p] = pack_f16(t0, t1);
               }
               st_chunk(sK + 2 * BLK, tid, c2, make_uint4(w4[0], w4[1], w4[2], w4[3]));
             }
@@ -297,7 +300,7 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
             const float p0 = (cb * 32 + e < nvalid) ? ex2(v[e] * sl2 - mb) : 0.0f;
             const float p1 = (cb * 32 + e + 1 < nvalid) ? ex2(v[e + 1] * sl2 - mb) : 0.0f;
             lsum += p0 + p1;
-            pk[e >> 1] = pack_bf16(p0, p1);
+            pk[e >> 1] = pack_f16(p0, p1);
           }
 #pragma unroll
           for (int k = 0; k < 4; ++k)
