@@ -141,6 +141,23 @@ QWM_API size_t qwm_fit_workspace_bytes(const qwm_config* cfg, int64_t N);
 QWM_API qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, void* centroids,
                              void* workspace, size_t workspace_bytes, void* stream);
 
+/* Allocation-free qwm_fit_centroids (the paper has no counterpart: this is an
+ * integration convenience).  For callers that cannot provide device scratch:
+ * a plain C host program holding only the tensors it was given, or an engine
+ * whose device memory is reserved by its own pool and which must not call
+ * cudaMalloc/cudaFree mid-generation (they can synchronise the device).  The
+ * k-means scratch lives in a static 16 MiB device array that every GPU which
+ * loads the library keeps until process exit; configurations needing more
+ * (fp32 + fp64 + count scratch of H*C*(12*d + 4) bytes, 256-byte padded per
+ * part) return QWM_ERR_CAPACITY.  Same arguments and results as
+ * qwm_fit_centroids without the workspace.  The first call on a device looks
+ * up the array's device address on the current device, so make that first
+ * call before any stream capture.  All calls share the one array: calls whose
+ * work overlaps on the GPU (different streams, or several host threads) race
+ * and give wrong centroids; serialise them. */
+QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, const void* x, int64_t N, void* centroids,
+                                             void* stream);
+
 /* Quantize one finished chunk and append it to the cache (Sec. 4.1 QSAC,
  * Sec. 2 Eq. 1-4 INT2 residuals, Sec. 4.2 Eq. 13/16 PSAC, App. D.1 packing).
  * k, v: bf16 [N][H][d], 1 <= N <= tokens_per_chunk.  k_centroids,

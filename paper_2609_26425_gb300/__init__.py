@@ -9,7 +9,7 @@ built, every call raises.
 
 Functions carry the C names:
   qwm_cache_bytes, qwm_fit_workspace_bytes, qwm_fit_centroids,
-  qwm_quantize_append, qwm_attend,
+  qwm_fit_centroids_noalloc, qwm_quantize_append, qwm_attend,
 and ``Cache`` wraps qwm_cache_init / qwm_cache_free / qwm_cache_status /
 qwm_cache_layout / qwm_cache_chunk_info.
 """
@@ -244,6 +244,23 @@ def qwm_fit_centroids(cfg: QwmConfig, x: torch.Tensor, centroids=None, workspace
         workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
     _check("qwm_fit_centroids", lib().qwm_fit_centroids(ct.byref(cfg), _ptr(x), N, _ptr(centroids),
                                                         _ptr(workspace), workspace.numel(), _stream()))
+    return centroids
+
+
+def qwm_fit_centroids_noalloc(cfg: QwmConfig, x: torch.Tensor, centroids=None) -> torch.Tensor:
+    """qwm_fit_centroids without a caller-provided workspace: the library keeps
+    the scratch in a static device array (see include/qwm.h for the limit and
+    the rule that overlapping calls race)."""
+    N = x.shape[0]
+    H, d, C = cfg.num_heads, cfg.head_dim, cfg.num_centroids
+    _bf16(x, (N, H, d), "x")
+    if centroids is None:
+        centroids = torch.empty(H, C, d, dtype=torch.bfloat16, device=x.device)
+    _bf16(centroids, (H, C, d), "centroids")
+    fn = lib().qwm_fit_centroids_noalloc
+    fn.argtypes = [_CFG, _P, ct.c_int64, _P, _P]
+    fn.restype = ct.c_int
+    _check("qwm_fit_centroids_noalloc", fn(ct.byref(cfg), _ptr(x), N, _ptr(centroids), _stream()))
     return centroids
 
 

@@ -7,6 +7,8 @@
 // index) and replaces each non-empty cluster by its member mean (member sums
 // accumulated in fp64, which is exact for bf16 members of ordinary range, so
 // the result does not depend on the order of the atomic adds).
+#include <mutex>
+
 #include "qwm_internal.cuh"
 
 namespace qwm {
@@ -98,3 +100,76 @@ cudaError_t launch_fit(const FitArgs& a, cudaStream_t st) {
 }
 
 }  // namespace qwm
+
+namespace qwm {
+
+// ----------------------------------------------------------------------------
+// Allocation-free variant of qwm_fit_centroids.
+//
+// Some callers cannot hand the library a scratch buffer: a plain C host
+// program that only owns the input and output tensors it was given, or an
+// inference engine whose device memory is already reserved by its own pool
+// and which must not call cudaMalloc/cudaFree in the middle of generation
+// (those calls can synchronise the whole device).  For them the k-means
+// scratch (fp32 centroids, fp64 member sums, member counts) lives in this
+// file-scope device array instead.
+// ----------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocFitScratchBytes = (size_t)16 << 20;  // 16 MiB per GPU that loads the library
+static __device__ __align__(256) uint8_t g_fit_scratch[kNoAllocFitScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_fit_scratch_mutex;
+void* g_fit_scratch_addr[kMaxDevices] = {};
+
+bool noalloc_cfg_ok(const qwm_config* c) {
+  return c->num_heads >= 1 && c->num_heads <= 4096 && c->head_dim == kHeadDim &&
+         (c->group_size == 32 || c->group_size == 64) && c->num_centroids >= 1 && c->num_centroids <= 256 &&
+         (c->psac_rank == 0 || c->psac_rank == 8 || c->psac_rank == 16 || c->psac_rank == 32) &&
+         c->num_candidates >= 1 && c->kmeans_iters >= 0;
+}
+
+}  // namespace
+}  // namespace qwm
+
+extern "C" QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, const void* x, int64_t N,
+                                                        void* centroids, void* stream) {
+  using namespace qwm;
+  if (!cfg || !x || !centroids || N < 1) return QWM_ERR_INVALID_ARG;
+  if (!noalloc_cfg_ok(cfg)) return QWM_ERR_UNSUPPORTED;
+  if (N > (int64_t)1 << 31) return QWM_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(x) & 15u) || (reinterpret_cast<uintptr_t>(centroids) & 15u))
+    return QWM_ERR_INVALID_ARG;
+  const size_t need = fit_workspace_bytes(cfg->num_heads, cfg->head_dim, cfg->num_centroids);
+  if (need > kNoAllocFitScratchBytes) return QWM_ERR_CAPACITY;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return QWM_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return QWM_ERR_UNSUPPORTED;
+  uint8_t* ws = nullptr;
+  {
+    // First call on a device: look up the device address of the array there
+    // (in host code its name is only a host-side stand-in).
+    std::lock_guard<std::mutex> lock(g_fit_scratch_mutex);
+    if (!g_fit_scratch_addr[dev]) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_fit_scratch) != cudaSuccess || !p) return QWM_ERR_CUDA;
+      g_fit_scratch_addr[dev] = p;
+    }
+    ws = static_cast<uint8_t*>(g_fit_scratch_addr[dev]);
+  }
+  FitArgs a{};
+  a.H = cfg->num_heads; a.d = cfg->head_dim; a.C = cfg->num_centroids; a.iters = cfg->kmeans_iters;
+  a.N = N;
+  a.x = static_cast<const __nv_bfloat16*>(x);
+  a.out = static_cast<__nv_bfloat16*>(centroids);
+  const size_t hcd = (size_t)a.H * a.C * a.d;
+  a.cent = reinterpret_cast<float*>(ws);
+  a.sums = reinterpret_cast<double*>(ws + round_up(hcd * 4, 256));
+  a.counts = reinterpret_cast<uint32_t*>(ws + round_up(hcd * 4, 256) + round_up(hcd * 8, 256));
+  // launch_fit writes every centroid before reading it and clears the sums
+  // and counts before each iteration, so nothing depends on what an earlier
+  // call left in the array.
+  return launch_fit(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
+}
+
