@@ -105,6 +105,17 @@ uint16_t oracle_f32_to_f16_ru(float x) {
   return f16_encode_exact(k * ulp);
 }
 
+/* Bit position of channel c's 2-bit code inside a token's packed codes
+ * (App. D.1 packs four INT2 codes per byte; the order inside is a reading):
+ * every 16 channels form one little-endian 32-bit word; inside it the even
+ * channel 2k sits at bits 2k and the odd channel 2k+1 at bits 16 + 2k.  Each
+ * byte still holds four codes (byte 0: channels 0,2,4,6; byte 1: 8..14 even;
+ * byte 2: 1,3,5,7; byte 3: 9..15 odd). */
+static int code_bit(int c) {
+  int j = c % 16;
+  return 32 * (c / 16) + 16 * (j & 1) + 2 * (j >> 1);
+}
+
 /* Round half to even (Eq. 1 rounding operator, reading: ties to even). */
 static float rint_even(float x) { return nearbyintf(x); }
 
@@ -279,8 +290,9 @@ static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uin
  *     lowers the approximated Query-weighted error; reading: the diagonal-w
  *     form of Eq. 8); otherwise codes and sigma are zero.
  *
- * Packing (App. D.1): channel c of a token goes to byte c/4, bits 2*(c%4);
- * group g's zero-point goes to byte g/4, bits 2*(g%4).
+ * Packing (App. D.1, four INT2 codes per byte): channel c's code sits at bit
+ * code_bit(c) of the token's d/4 code bytes (see code_bit; d must be a
+ * multiple of 16); group g's zero-point goes to byte g/4, bits 2*(g%4).
  *
  * Outputs ([N][H][...] token-major; pointers marked optional may be NULL):
  *   ids[N][H] u8, codes[N][H][d/4] u8, scales[N][H][d/G] fp16 bits,
@@ -305,7 +317,7 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
                     int8_t* coef, uint16_t* sigma, uint8_t* kept,
                     float* khat0, int32_t* cand, float* m_topm, float* m_sel, float* m_psac,
                     float* dq_out, float* s_out, int nthreads) {
-  if (H <= 0 || d <= 0 || d > 256 || C <= 0 || C > 256 || G <= 0 || d % G || d % 4 || r < 0 || M <= 0 || N < 0)
+  if (H <= 0 || d <= 0 || d > 256 || C <= 0 || C > 256 || G <= 0 || d % G || d % 16 || r < 0 || M <= 0 || N < 0)
     return ORC_EINVAL;
   if (!x || !cent || !ids || !codes || !scales || !zeros) return ORC_EINVAL;
   const int ng = d / G;
@@ -434,7 +446,8 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
       float s = oracle_f16_to_f32(sb);
       for (int c = g * G; c < (g + 1) * G; ++c) {
         int q = qv[c - g * G];
-        cd[c / 4] |= (uint8_t)(q << (2 * (c % 4)));
+        int bit = code_bit(c);
+        cd[bit / 8] |= (uint8_t)(q << (bit % 8));
         float deq = (float)(q - z) * s;
         k0[c] = oracle_bf16_to_f32(mu[c]) + deq;
       }
@@ -543,7 +556,8 @@ int oracle_dequant(int H, int d, int C, int G, int r, int64_t N, const uint16_t*
       const uint16_t* mu = cent + ((size_t)h * C + id) * d;
       for (int c = 0; c < d; ++c) {
         int g = c / G;
-        int q = (codes[th * (d / 4) + c / 4] >> (2 * (c % 4))) & 3;
+        int bit = code_bit(c);
+        int q = (codes[th * (d / 4) + bit / 8] >> (bit % 8)) & 3;
         int z = (zeros[th * zb + g / 4] >> (2 * (g % 4))) & 3;
         double s = (double)oracle_f16_to_f32(scales[th * ng + g]);
         double v = (double)oracle_bf16_to_f32(mu[c]) + s * (double)(q - z);

@@ -25,12 +25,20 @@ def bf(x):
     return b
 
 
+def code_bit(c):
+    """Bit of channel c's code (App. D.1 packing reading: 16-channel little-endian
+    words, even channel 2k at bit 2k, odd channel 2k+1 at bit 16+2k)."""
+    j = c % 16
+    return 32 * (c // 16) + 16 * (j & 1) + 2 * (j >> 1)
+
+
 def unpack2(bytes_, n):
     b = np.asarray(bytes_, np.uint8)
-    out = np.zeros(b.shape[:-1] + (b.shape[-1] * 4,), np.int64)
-    for i in range(4):
-        out[..., i::4] = (b >> (2 * i)) & 3
-    return out[..., :n]
+    out = np.zeros(b.shape[:-1] + (n,), np.int64)
+    for c in range(n):
+        bit = code_bit(c)
+        out[..., c] = (b[..., bit // 8] >> (bit % 8)) & 3
+    return out
 
 
 def f16(bits):
@@ -105,10 +113,10 @@ def test_int2_zero_and_constant_groups(orc):
 
 
 def test_packing_layout(orc):
-    """Channel c -> byte c/4 bits 2(c%4); zero-point g -> byte g/4 bits 2(g%4) (App. D.1)."""
+    """Four INT2 codes per byte (App. D.1): channel c at bit code_bit(c);
+    zero-point g at byte g/4, bits 2(g%4)."""
     d, G = 128, 32
     s = 0.25
-    # group g holds the pattern (c + g) % 4 - z with a chosen zero point z = g % 4 ... kept on grid
     x = np.zeros((1, 1, d), np.float32)
     want_codes = np.zeros(d, np.int64)
     want_z = []
@@ -120,12 +128,14 @@ def test_packing_layout(orc):
         want_codes[g * G:(g + 1) * G] = q
         x[0, 0, g * G:(g + 1) * G] = (q - z) * s
     o = orc.quantize(bf(x), np.zeros((1, 1, d), np.uint16), G=G, r=0, M=1, is_key=True)
-    packed = np.zeros(d // 4, np.uint8)
+    words = np.zeros(d // 16, np.uint32)
     for c in range(d):
-        packed[c // 4] |= np.uint8(want_codes[c] << (2 * (c % 4)))
-    assert np.array_equal(o["codes"][0, 0], packed)
+        w, j = divmod(c, 16)
+        words[w] |= np.uint32(want_codes[c] << (2 * (j >> 1) + 16 * (j & 1)))
+    assert np.array_equal(o["codes"][0, 0], words.view(np.uint8))
     zbyte = sum(z << (2 * g) for g, z in enumerate(want_z))
     assert o["zeros"][0, 0, 0] == zbyte
+    assert np.array_equal(unpack2(o["codes"], d)[0, 0], want_codes)
 
 
 # --------------------------------------------------------------------- QSAC
