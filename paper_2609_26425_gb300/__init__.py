@@ -187,8 +187,8 @@ class Cache:
         """Copy chunk i (0 = oldest held) back to the host as token-major numpy
         arrays (layout only; no arithmetic): ids [N][H], codes [N][H][d/4],
         scales [N][H][d/G] (binary16 bits), zeros [N][H][zb], coef [N][H][r],
-        sigma [N][H] (binary16 bits), k_tab / v_tab [H][C][d] and U [H][d][r]
-        (bf16 bits)."""
+        sigma [N][H] (binary16 bits), k_tab / v_tab [H][C][d] (binary16 bits,
+        the tables as stored in the slot) and U [H][d][r] (bf16 bits)."""
         slot, N = self.chunk_info(i)
         lay = self.layout()
         cfg = self.cfg

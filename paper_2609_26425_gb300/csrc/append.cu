@@ -75,11 +75,16 @@ __global__ void __launch_bounds__(NT, 1) append_kernel(const AppendArgs a) {
   s.t0 = reinterpret_cast<float*>(p); p += NW * 128 * 4;
   s.cand = reinterpret_cast<int*>(p);
 
-  // The chunk's own tables travel with the slot (one CTA per head and K/V).
+  // The chunk's own tables travel with the slot (one CTA per head and K/V),
+  // stored as binary16 (exact for bf16 values in the binary16 range), the
+  // operand type of the attention kernel's tensor-core path.
   if (blockIdx.x == 0) {
-    const uint4* src = reinterpret_cast<const uint4*>(tab);
-    uint4* dst = reinterpret_cast<uint4*>(head + (is_key ? L.ktab : L.vtab));
-    for (int i = tid; i < C * 16; i += NT) dst[i] = src[i];
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
+    __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
+    for (int i = tid; i < C * 64; i += NT) {
+      const uint32_t pr = src[i];
+      dst[i] = __floats2half2_rn(bf_lo(pr), bf_hi(pr));
+    }
     if (psac) {
       __nv_bfloat16* ut = reinterpret_cast<__nv_bfloat16*>(head + L.ut);
       const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * r;
@@ -243,7 +248,16 @@ __global__ void __launch_bounds__(NT, 1) append_kernel(const AppendArgs a) {
     const int64_t o_scales = is_key ? L.k_scales : L.v_scales;
     const int64_t o_ids = is_key ? L.k_ids : L.v_ids;
     const int64_t o_zeros = is_key ? L.k_zeros : L.v_zeros;
-    tb[o_codes + rowi * 32 + lane] = (uint8_t)cbyte;
+    // Packed codes: 16 channels per little-endian 32-bit word, even channel 2k
+    // at bits 2k, odd channel 2k+1 at bits 16 + 2k (four codes per byte).
+    // This lane holds channels 4*lane .. 4*lane+3 = word lane/4, pairs m, m+1
+    // with m = 2*(lane % 4).
+    const int csh = 4 * (lane & 3);
+    uint32_t word = ((cbyte & 3u) << csh) | (((cbyte >> 2) & 3u) << (16 + csh)) |
+                    (((cbyte >> 4) & 3u) << (csh + 2)) | (((cbyte >> 6) & 3u) << (16 + csh + 2));
+    word |= __shfl_xor_sync(0xFFFFFFFFu, word, 1);
+    word |= __shfl_xor_sync(0xFFFFFFFFu, word, 2);
+    if ((lane & 3) == 0) *reinterpret_cast<uint32_t*>(tb + o_codes + rowi * 32 + lane) = word;
     if (lane % glanes == 0)
       reinterpret_cast<__half*>(tb + o_scales + (int64_t)rowi * ng * 2)[lane / glanes] = sh;
     if (lane == 0) {

@@ -33,6 +33,12 @@ def dev(t):
     return t.to("cuda").contiguous()
 
 
+def f16_bits(bf16_bits):
+    """bf16 bit patterns -> binary16 bit patterns of the same values (torch conversion)."""
+    t = synth.from_bits(bf16_bits).to(torch.float16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
 def strided_centroids(x_bits, C):
     """Generator-side centroid table: tokens floor(j*N/C) of the chunk (no arithmetic)."""
     N = x_bits.shape[0]
@@ -72,7 +78,7 @@ def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None
     ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub)
     sk = compare_packed(dec, ko, kb, kc, G=G, r=r, M=M, is_key=True, w=w, U_bits=Ub)
     sv = compare_packed(dec, vo, vb, vc, G=G, r=r, M=M, is_key=False, prefix="v_")
-    assert np.array_equal(dec["k_tab"], kc) and np.array_equal(dec["v_tab"], vc)
+    assert np.array_equal(dec["k_tab"], f16_bits(kc)) and np.array_equal(dec["v_tab"], f16_bits(vc))
     if Ub is not None:
         assert np.array_equal(dec["U"], Ub)
     return sk, sv
