@@ -416,11 +416,11 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
             for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
               for (int ks = 0; ks < 4; ++ks)
-                umma_bf16(tS, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
+                umma_ss(tS, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
                           desc_sw128(aK + (2 * st + kb) * BLK + ks * 32), idS, (kb | ks) != 0);
             if (U.psac)
               for (int ks = 0; ks < rpad / 16; ++ks)
-                umma_bf16(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32),
+                umma_ss(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32),
                           idS, 1u);
             umma_commit(bar(B_SFULL + i));
           }

@@ -170,7 +170,7 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool b_mn_major, 
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T, one CTA, issued by one thread.
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+__device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                           uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"

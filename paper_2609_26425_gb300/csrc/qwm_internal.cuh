@@ -89,6 +89,7 @@ struct AppendArgs {
   int M;                       // candidates (clamped to C)
 };
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
+cudaError_t launch_append_generic(const AppendArgs& a, cudaStream_t s);
 
 struct AttendSlots {
   int32_t n;

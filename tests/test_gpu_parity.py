@@ -92,6 +92,8 @@ def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None
     (2, 200, 8, 32, 16, 8, True, True),       # exhaustive QSAC (M = C)
     (2, 129, 64, 64, 0, 4, True, False),      # PSAC disabled by rank 0
     (1, 1, 4, 32, 8, 4, True, True),          # a single token
+    (2, 150, 64, 32, 16, 12, True, True),     # 8 < M < C: the generic kernel
+    (2, 300, 256, 64, 32, 2, True, True),     # G = 64 with the largest table
 ])
 def test_append_parity(H, N, C, G, r, M, use_w, use_U):
     sk, sv = run_append_case(H, N, C, G, r, M, use_w, use_U, seed=H * 1000 + N)
