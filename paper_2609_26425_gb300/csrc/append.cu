@@ -352,8 +352,8 @@ __global__ void __launch_bounds__(NT, 2) append_kernel(const AppendArgs a) {
 #pragma unroll
       for (int g = 0; g < 4; ++g) {
         if (g < ng) {
-          const float R = __fsub_rn(mx[g], mn[g]);
-          S = __fadd_rn(S, __fmul_rn(sWg[g], __fmul_rn(R, R)));
+          const float Rg = __fsub_rn(mx[g], mn[g]);
+          S = __fadd_rn(S, __fmul_rn(sWg[g], __fmul_rn(Rg, Rg)));
         }
       }
       if (S < bestS || (S == bestS && j < bestj)) { bestS = S; bestj = j; }

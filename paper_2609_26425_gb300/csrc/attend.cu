@@ -63,46 +63,118 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+__device__ __forceinline__ uint32_t ex2_f16x2(uint32_t x) {
+  uint32_t y;
+  asm("ex2.approx.f16x2 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+// (a, b) = (a, b) * (s, s) + (c, c) as one packed f32x2 fma.
+__device__ __forceinline__ void fma2(float& a, float& b, uint64_t ss, uint64_t cc) {
+  uint64_t x;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(x) : "f"(a), "f"(b));
+  asm("fma.rn.f32x2 %0, %0, %1, %2;" : "+l"(x) : "l"(ss), "l"(cc));
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(x));
+}
+__device__ __forceinline__ uint64_t splat2(float a) {
+  uint64_t x;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(x) : "f"(a));
+  return x;
+}
+// acc + (low half of h2 as f16), acc + (high half), in one mixed-precision add each.
+__device__ __forceinline__ float add_f16lo(float acc, uint32_t h2) {
+  float r;
+  asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.f16 %0, lo, %2;\n\t}" : "=f"(r) : "r"(h2), "f"(acc));
+  return r;
+}
+__device__ __forceinline__ float add_f16hi(float acc, uint32_t h2) {
+  float r;
+  asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.f16 %0, hi, %2;\n\t}" : "=f"(r) : "r"(h2), "f"(acc));
+  return r;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float m;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(m) : "f"(a), "f"(b), "f"(c));
+  return m;
+}
+
 __device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
 __device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
+
+// The packed fields of one cache row, loaded one tile ahead of their use so
+// that their latency overlaps the rebuild of the current tile.
+struct RowPack {
+  uint4 c0, c1;   // 128 INT2 codes
+  uint32_t idz;   // centroid id | zero-point byte << 8
+  uint2 sc;       // group scales (binary16), d/G <= 4 of them
+  uint4 cf0, cf1; // PSAC INT8 codes (Keys, r <= 32)
+  uint32_t sg;    // PSAC row scale (binary16 bits)
+};
+
+__device__ __forceinline__ RowPack load_pack(const uint8_t* tb, int row, int64_t o_codes, int64_t o_scales,
+                                             int64_t o_ids, int64_t o_zeros, int zb, int ng, bool with_psac,
+                                             int64_t o_coef, int64_t o_sigma, int r) {
+  RowPack p;
+  p.c0 = ldg16(tb + o_codes + row * 32);
+  p.c1 = ldg16(tb + o_codes + row * 32 + 16);
+  p.idz = (uint32_t)tb[o_ids + row] | ((uint32_t)tb[o_zeros + (int64_t)row * zb] << 8);
+  const uint8_t* sp = tb + o_scales + (int64_t)row * ng * 2;
+  p.sc = ng == 4 ? __ldg(reinterpret_cast<const uint2*>(sp)) : make_uint2(__ldg(reinterpret_cast<const uint32_t*>(sp)), 0u);
+  p.cf0 = make_uint4(0, 0, 0, 0);
+  p.cf1 = make_uint4(0, 0, 0, 0);
+  p.sg = 0;
+  if (with_psac) {
+    const uint8_t* cp = tb + o_coef + (int64_t)row * r;
+    if (r == 8) {
+      const uint2 v = __ldg(reinterpret_cast<const uint2*>(cp));
+      p.cf0 = make_uint4(v.x, v.y, 0, 0);
+    } else {
+      p.cf0 = ldg16(cp);
+      if (r == 32) p.cf1 = ldg16(cp + 16);
+    }
+    p.sg = __ldg(reinterpret_cast<const unsigned short*>(tb + o_sigma + row * 2));
+  }
+  return p;
+}
 
 // One row of K_hat0 or V_hat: mu_id + s_g (q - z_g), computed as packed f16
 // pairs: the two codes of channels (2k, 2k+1) sit at bits 2k and 16 + 2k of
 // their 16-channel word, so (word >> 2k) & 0x00030003 | 0x64006400 is the f16
 // pair (1024 + q, 1024 + q'), (1024 + q) - (1024 + z) = q - z exactly, and one
 // f16 fma adds the centroid with a single rounding.  The table is binary16.
-__device__ __forceinline__ void dequant_row(uint8_t* dst, int row, const uint8_t* tb, int64_t o_codes,
-                                            int64_t o_scales, int64_t o_ids, int64_t o_zeros, int zb, int ng,
-                                            int gshift, const uint8_t* tab) {
-  const uint4 c0 = ldg16(tb + o_codes + row * 32);
-  const uint4 c1 = ldg16(tb + o_codes + row * 32 + 16);
-  const uint32_t cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-  const int id = tb[o_ids + row];
-  const uint32_t zbyte = tb[o_zeros + (int64_t)row * zb];
-  const __half* sp = reinterpret_cast<const __half*>(tb + o_scales + (int64_t)row * ng * 2);
+__device__ __forceinline__ void dequant_row(uint8_t* dst, int row, const RowPack& p, int ng, int gshift,
+                                            const uint8_t* tab) {
+  const uint32_t cw[8] = {p.c0.x, p.c0.y, p.c0.z, p.c0.w, p.c1.x, p.c1.y, p.c1.z, p.c1.w};
+  const uint32_t zbyte = (p.idz >> 8) & 0xFFu;
+  const uint32_t sw[2] = {p.sc.x, p.sc.y};
   __half2 s2[4], z2[4];
 #pragma unroll
   for (int g = 0; g < 4; ++g) {
-    const __half sg = g < ng ? sp[g] : __ushort_as_half(0);
-    s2[g] = __halves2half2(sg, sg);
+    const uint32_t sbits = g < ng ? ((sw[g >> 1] >> (16 * (g & 1))) & 0xFFFFu) : 0u;
+    s2[g] = u2h(sbits | (sbits << 16));
     const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
     z2[g] = u2h(zz | (zz << 16));
   }
-  const uint8_t* mu = tab + (int64_t)id * 256;
+  const uint8_t* mu = tab + (int64_t)(p.idz & 0xFFu) * 256;
 #pragma unroll
-  for (int ch = 0; ch < 16; ++ch) {
-    const int g = (ch * 8) >> gshift;
-    const uint32_t word = cw[ch >> 1];
-    const uint4 m = ldg16(mu + ch * 16);
-    const uint32_t mw[4] = {m.x, m.y, m.z, m.w};
-    uint32_t ow[4];
+  for (int half = 0; half < 2; ++half) {
+    uint4 mrow[8];  // half a centroid row in flight at once
 #pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      const int k = 4 * (ch & 1) + p;
-      const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
-      ow[p] = h2u(__hfma2(__hsub2(u2h(qq), z2[g]), s2[g], u2h(mw[p])));
+    for (int i = 0; i < 8; ++i) mrow[i] = ldg16(mu + (half * 8 + i) * 16);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int ch = half * 8 + i;
+      const int g = (ch * 8) >> gshift;
+      const uint32_t word = cw[ch >> 1];
+      const uint32_t mw[4] = {mrow[i].x, mrow[i].y, mrow[i].z, mrow[i].w};
+      uint32_t ow[4];
+#pragma unroll
+      for (int q2 = 0; q2 < 4; ++q2) {
+        const int k = 4 * (ch & 1) + q2;
+        const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+        ow[q2] = h2u(__hfma2(__hsub2(u2h(qq), z2[g]), s2[g], u2h(mw[q2])));
+      }
+      st_chunk(dst, row, ch, make_uint4(ow[0], ow[1], ow[2], ow[3]));
     }
-    st_chunk(dst, row, ch, make_uint4(ow[0], ow[1], ow[2], ow[3]));
   }
 }
 
@@ -134,6 +206,25 @@ __device__ __forceinline__ Unit unit_at(const AttendArgs& a, const AttendSlots& 
   }
   return x;
 }
+
+// Walks the KV tiles of every unit (cached chunks in order, then the active
+// chunk) in the order all roles process them.
+struct TileCursor {
+  int u, tl, n_units, ntiles;
+  Unit U;
+  __device__ __forceinline__ void init(const AttendArgs& a, const AttendSlots& S, int h, int nu) {
+    u = 0; tl = 0; n_units = nu; ntiles = 0;
+    if (nu > 0) { U = unit_at(a, S, 0, h); ntiles = (U.ntok + 127) / 128; }
+  }
+  __device__ __forceinline__ bool valid() const { return u < n_units; }
+  __device__ __forceinline__ void next(const AttendArgs& a, const AttendSlots& S, int h) {
+    if (++tl >= ntiles) {
+      tl = 0;
+      if (++u < n_units) { U = unit_at(a, S, u, h); ntiles = (U.ntok + 127) / 128; }
+    }
+  }
+  __device__ __forceinline__ int nvalid() const { return min(128, U.ntok - tl * 128); }
+};
 
 // Q_i U_r of one query row (fp32 sums of bf16 products), as f16 into the
 // shared Q U_r block at columns [i*rpad, i*rpad + rpad).
@@ -256,9 +347,14 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
 #pragma unroll
         for (int cb = 0; cb < 4; ++cb) {
           tmem_ld32(tS + cb * 32, v);
+          if (nvalid == 128) {
 #pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (cb * 32 + e < nvalid) mt = fmaxf(mt, v[e]);
+            for (int e = 0; e < 32; e += 2) mt = fmax3(mt, v[e], v[e + 1]);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (cb * 32 + e < nvalid) mt = fmaxf(mt, v[e]);
+          }
         }
         const float m_new = fmaxf(m_run, mt);
         const bool need = (m_new - m_run) * sl2 > kTauLog2;
@@ -280,20 +376,29 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
           }
         }
         const float mb = m_run * sl2;
-        float lsum = 0.0f;
+        const uint64_t SL = splat2(sl2), MB = splat2(-mb);
+        float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
         for (int cb = 0; cb < 4; ++cb) {
           tmem_ld32(tS + cb * 32, v);
           uint32_t pk[16];
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            const float p0 = (cb * 32 + e < nvalid) ? ex2(v[e] * sl2 - mb) : 0.0f;
-            const float p1 = (cb * 32 + e + 1 < nvalid) ? ex2(v[e + 1] * sl2 - mb) : 0.0f;
-            lsum += p0 + p1;
-            pk[e >> 1] = pack_f16(p0, p1);
+            // x = s * scale * log2(e) - m, exp2 of the f16 pair in one MUFU op;
+            // P is the f16 MMA operand and the row sum adds exactly those values.
+            float x0 = v[e], x1 = v[e + 1];
+            fma2(x0, x1, SL, MB);
+            if (nvalid < 128) {
+              if (cb * 32 + e >= nvalid) x0 = -INFINITY;
+              if (cb * 32 + e + 1 >= nvalid) x1 = -INFINITY;
+            }
+            const uint32_t p2 = ex2_f16x2(pack_f16(x0, x1));
+            ls[(e >> 1) & 3] = add_f16lo(add_f16hi(ls[(e >> 1) & 3], p2), p2);
+            pk[e >> 1] = p2;
           }
           tmem_st16(tS + cb * 16, pk);  // P (f16 pairs) over the columns already read
         }
+        const float lsum = (ls[0] + ls[1]) + (ls[2] + ls[3]);
         tmem_wait_st();
         l_run += lsum;
         tc_fence_before();
@@ -335,111 +440,132 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
     // ------------------------------------------------------------ dequant K (warps 8-11) / V (12-15)
     const bool isK = warp < W_DQV;
     const int row = tid & 127;
+    const int64_t o_codes = isK ? L.k_codes : L.v_codes, o_scales = isK ? L.k_scales : L.v_scales;
+    const int64_t o_ids = isK ? L.k_ids : L.v_ids, o_zeros = isK ? L.k_zeros : L.v_zeros;
+    // The packed fields of tile j+1 are loaded while tile j is rebuilt.
+    TileCursor cur;
+    cur.init(a, S, h, n_units);
+    RowPack nxt{};
+    if (cur.valid() && cur.U.hb && row < cur.nvalid())
+      nxt = load_pack(cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes, row, o_codes, o_scales, o_ids, o_zeros,
+                      L.zb, L.ng, isK && cur.U.psac, L.k_coef, L.k_sigma, r);
     uint32_t jt = 0;
     bool ok = true;
-    for (int u = 0; u < n_units && ok; ++u) {
-      const Unit U = unit_at(a, S, u, h);
-      const int ntiles = (U.ntok + 127) / 128;
-      for (int tl = 0; tl < ntiles; ++tl, ++jt) {
-        const int st = jt & 1;
-        const uint32_t ph = (jt >> 1) & 1;
-        const int nvalid = min(128, U.ntok - tl * 128);
-        const bool rvalid = row < nvalid;
-        if (!mbar_wait(bar((isK ? B_KEMPTY : B_VEMPTY) + st), ph ^ 1)) {
-          ok = false;
-          break;
-        }
-        uint8_t* dst = sm + (isK ? OFF_K : OFF_V) + st * 2 * BLK;
-        if (!rvalid) {
-          zero_row(dst, row, 0, 16);
-        } else if (!U.hb) {
-          const __nv_bfloat16* src = (isK ? a.kcur : a.vcur) + ((size_t)(tl * 128 + row) * H + h) * 128;
-          copy_row(dst, row, src);
-        } else {
-          const uint8_t* tb = U.hb + L.tiles_off + (int64_t)tl * L.tile_bytes;
-          if (isK)
-            dequant_row(dst, row, tb, L.k_codes, L.k_scales, L.k_ids, L.k_zeros, L.zb, L.ng, gshift, U.hb + L.ktab);
-          else
-            dequant_row(dst, row, tb, L.v_codes, L.v_scales, L.v_ids, L.v_zeros, L.zb, L.ng, gshift, U.hb + L.vtab);
-        }
-        if (isK && U.psac) {
-          uint8_t* sC = sm + OFF_C;
-          const int ch0 = (st * rpad) / 8;
-          if (rvalid) {
-            const uint8_t* tb = U.hb + L.tiles_off + (int64_t)tl * L.tile_bytes;
-            const int8_t* cp = reinterpret_cast<const int8_t*>(tb + L.k_coef + (int64_t)row * r);
-            const float sg = __half2float(*reinterpret_cast<const __half*>(tb + L.k_sigma + row * 2));
-            for (int c2 = 0; c2 * 8 < rpad; ++c2) {
+    while (cur.valid()) {
+      const RowPack pk = nxt;
+      TileCursor nc = cur;
+      nc.next(a, S, h);
+      if (nc.valid() && nc.U.hb && row < nc.nvalid())
+        nxt = load_pack(nc.U.hb + L.tiles_off + (int64_t)nc.tl * L.tile_bytes, row, o_codes, o_scales, o_ids,
+                        o_zeros, L.zb, L.ng, isK && nc.U.psac, L.k_coef, L.k_sigma, r);
+      const int st = jt & 1;
+      const uint32_t ph = (jt >> 1) & 1;
+      const bool rvalid = row < cur.nvalid();
+      if (!mbar_wait(bar((isK ? B_KEMPTY : B_VEMPTY) + st), ph ^ 1)) {
+        ok = false;
+        break;
+      }
+      uint8_t* dst = sm + (isK ? OFF_K : OFF_V) + st * 2 * BLK;
+      if (!rvalid) {
+        zero_row(dst, row, 0, 16);
+      } else if (!cur.U.hb) {
+        copy_row(dst, row, (isK ? a.kcur : a.vcur) + ((size_t)(cur.tl * 128 + row) * H + h) * 128);
+      } else {
+        dequant_row(dst, row, pk, L.ng, gshift, cur.U.hb + (isK ? L.ktab : L.vtab));
+      }
+      if (isK && cur.U.psac) {
+        uint8_t* sC = sm + OFF_C;
+        const int ch0 = (st * rpad) / 8;
+        if (rvalid) {
+          const float sg = __half2float(__ushort_as_half((unsigned short)pk.sg));
+          const uint32_t cwd[8] = {pk.cf0.x, pk.cf0.y, pk.cf0.z, pk.cf0.w, pk.cf1.x, pk.cf1.y, pk.cf1.z, pk.cf1.w};
+#pragma unroll
+          for (int c2 = 0; c2 < 4; ++c2) {
+            if (c2 * 8 < rpad) {
               uint32_t w4[4];
 #pragma unroll
-              for (int p = 0; p < 4; ++p) {
-                const int j = c2 * 8 + 2 * p;
-                w4[p] = pack_f16(j < r ? (float)cp[j] * sg : 0.0f, j + 1 < r ? (float)cp[j + 1] * sg : 0.0f);
+              for (int q2 = 0; q2 < 4; ++q2) {
+                const int j = c2 * 8 + 2 * q2;
+                const uint32_t wd = cwd[j >> 2];
+                const float t0 = j < r ? (float)(int8_t)(wd >> (8 * (j & 3))) * sg : 0.0f;
+                const float t1 = j + 1 < r ? (float)(int8_t)(wd >> (8 * ((j + 1) & 3))) * sg : 0.0f;
+                w4[q2] = pack_f16(t0, t1);
               }
               st_chunk(sC, row, ch0 + c2, make_uint4(w4[0], w4[1], w4[2], w4[3]));
             }
-          } else {
-            zero_row(sC, row, ch0, rpad / 8);
           }
+        } else {
+          zero_row(sC, row, ch0, rpad / 8);
         }
-        fence_proxy_async_smem();
-        mbar_arrive(bar((isK ? B_KFULL : B_VFULL) + st));
       }
+      fence_proxy_async_smem();
+      mbar_arrive(bar((isK ? B_KFULL : B_VFULL) + st));
+      cur = nc;
+      ++jt;
     }
     if (!ok) *s_err = 1;
   } else {
     // ------------------------------------------------------------ MMA issue (one thread)
+    // Order per KV tile j: P0 V(j), S0(j+1), P1 V(j), S1(j+1), so that the
+    // softmax of Q tile 0 on tile j+1 overlaps the softmax of Q tile 1 on
+    // tile j (S_i(j+1) reuses the TMEM columns of P_i(j) after P_i V(j) has
+    // read them: MMAs of one thread run in issue order).
     if (lane == 0) {
       const uint32_t aQ = smem_u32(sm + OFF_Q), aQU = smem_u32(sm + OFF_QU);
       const uint32_t aK = smem_u32(sm + OFF_K), aC = smem_u32(sm + OFF_C), aV = smem_u32(sm + OFF_V);
       constexpr uint32_t idS = idesc_f16(128, 128, false);
       constexpr uint32_t idPV = idesc_f16(128, 64, true);
-      uint32_t jt = 0, qph = 0;
+      int total = 0;
+      for (int u = 0; u < n_units; ++u) total += (unit_at(a, S, u, h).ntok + 127) / 128;
+      TileCursor sc;  // next tile to issue S for
+      sc.init(a, S, h, n_units);
+      uint32_t sjt = 0, qph[2] = {0, 0};
       bool ok = true;
-      for (int u = 0; u < n_units && ok; ++u) {
-        const Unit U = unit_at(a, S, u, h);
-        const int ntiles = (U.ntok + 127) / 128;
-        for (int tl = 0; tl < ntiles; ++tl, ++jt) {
-          const int st = jt & 1;
-          const uint32_t ph = (jt >> 1) & 1;
-          if (tl == 0 && (u == 0 || U.psac)) {
-            ok = mbar_wait(bar(B_QU + 0), qph) && mbar_wait(bar(B_QU + 1), qph);
-            qph ^= 1;
-            if (!ok) break;
-          }
-          if (!(ok = mbar_wait(bar(B_KFULL + st), ph))) break;
-          tc_fence_after();
+      auto issue_S = [&](int i) -> bool {
+        const int st = sjt & 1;
+        const uint32_t ph = (sjt >> 1) & 1;
+        if (sc.tl == 0 && (sc.u == 0 || sc.U.psac)) {
+          if (!mbar_wait(bar(B_QU + i), qph[i])) return false;
+          qph[i] ^= 1;
+        }
+        if (i == 0 && !mbar_wait(bar(B_KFULL + st), ph)) return false;
+        tc_fence_after();
+        const uint32_t tS = tbase + 128 * i;
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            const uint32_t tS = tbase + 128 * i;
+        for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
-            for (int kb = 0; kb < 2; ++kb)
-#pragma unroll
-              for (int ks = 0; ks < 4; ++ks)
-                umma_ss(tS, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
-                          desc_sw128(aK + (2 * st + kb) * BLK + ks * 32), idS, (kb | ks) != 0);
-            if (U.psac)
-              for (int ks = 0; ks < rpad / 16; ++ks)
-                umma_ss(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32),
-                          idS, 1u);
-            umma_commit(bar(B_SFULL + i));
-          }
+          for (int ks = 0; ks < 4; ++ks)
+            umma_ss(tS, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32), desc_sw128(aK + (2 * st + kb) * BLK + ks * 32),
+                    idS, (kb | ks) != 0);
+        if (sc.U.psac)
+          for (int ks = 0; ks < rpad / 16; ++ks)
+            umma_ss(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32), idS, 1u);
+        umma_commit(bar(B_SFULL + i));
+        if (i == 1) {
           umma_commit(bar(B_KEMPTY + st));
-          if (!(ok = mbar_wait(bar(B_VFULL + st), ph))) break;
+          sc.next(a, S, h);
+          ++sjt;
+        }
+        return true;
+      };
+      if (total > 0) ok = issue_S(0) && issue_S(1);
+      for (int jt = 0; jt < total && ok; ++jt) {
+        const int st = jt & 1;
+        const uint32_t ph = (jt >> 1) & 1;
+        if (!(ok = mbar_wait(bar(B_VFULL + st), ph))) break;
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            if (!(ok = mbar_wait(bar(B_PFULL + i), jt & 1))) break;
-            tc_fence_after();
-            const uint32_t tP = tbase + 128 * i, tO = tbase + 256 + 128 * i;
+        for (int i = 0; i < 2; ++i) {
+          if (!(ok = mbar_wait(bar(B_PFULL + i), jt & 1))) break;
+          tc_fence_after();
+          const uint32_t tP = tbase + 128 * i, tO = tbase + 256 + 128 * i;
 #pragma unroll
-            for (int ks = 0; ks < 8; ++ks)
+          for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
-              for (int nh = 0; nh < 2; ++nh)
-                umma_ts(tO + 64 * nh, tP + 8 * ks, desc_sw128(aV + (2 * st + nh) * BLK + ks * 2048), idPV,
-                        (jt > 0 || ks > 0) ? 1u : 0u);
-          }
-          if (!ok) break;
-          umma_commit(bar(B_VEMPTY + st));
+            for (int nh = 0; nh < 2; ++nh)
+              umma_ts(tO + 64 * nh, tP + 8 * ks, desc_sw128(aV + (2 * st + nh) * BLK + ks * 2048), idPV,
+                      (jt > 0 || ks > 0) ? 1u : 0u);
+          if (i == 1) umma_commit(bar(B_VEMPTY + st));
+          if (jt + 1 < total && !(ok = issue_S(i))) break;
         }
       }
       umma_commit(bar(B_OFINAL));
