@@ -248,7 +248,7 @@ def run_gpu(args, wl, rank, world):
     res = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": wl.name, "heads": H, "head_dim": wl.head_dim, "chunk_tokens": N,
                    "cached_tokens": wl.cache_tokens, "active_tokens": N, "query_tokens": N,
                    "centroids": C, "group_size": G, "psac_rank": r, "candidates": M,
