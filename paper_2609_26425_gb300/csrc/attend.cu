@@ -97,6 +97,13 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return m;
 }
 
+// 32-byte read-only global load (address 32-byte aligned).
+__device__ __forceinline__ void ldg32B(const void* p, uint32_t (&r)[8]) {
+  asm volatile("ld.global.nc.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+               : "l"(p));
+}
+
 __device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
 __device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
 
@@ -439,63 +446,138 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
   } else if (warp < W_MMA) {
     // ------------------------------------------------------------ dequant K (warps 8-11) / V (12-15)
     const bool isK = warp < W_DQV;
-    const int row = tid & 127;
     const int64_t o_codes = isK ? L.k_codes : L.v_codes, o_scales = isK ? L.k_scales : L.v_scales;
     const int64_t o_ids = isK ? L.k_ids : L.v_ids, o_zeros = isK ? L.k_zeros : L.v_zeros;
-    // The packed fields of tile j+1 are loaded while tile j is rebuilt.
+    // Four lanes per row: lane q of a quad rebuilds channels 16q..16q+15 and
+    // 64+16q..64+16q+15 of its row (chunks 2q, 2q+1, 8+2q, 9+2q), reading
+    // 32-byte slices, so one warp-wide load touches 8 centroid rows (8 cache
+    // lines) instead of 32.  Warp w of the group covers rows 32w..32w+31 in
+    // four passes of 8 rows, two passes per round of loads.  The rows'
+    // centroid ids and zero-points of the next tile are loaded one tile ahead.
+    const int q = lane & 3, rr = lane >> 2;
+    const int wrow = (warp & 3) * 32 + rr;  // row of pass p: wrow + 8p
     TileCursor cur;
     cur.init(a, S, h, n_units);
-    RowPack nxt{};
-    if (cur.valid() && cur.U.hb && row < cur.nvalid())
-      nxt = load_pack(cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes, row, o_codes, o_scales, o_ids, o_zeros,
-                      L.zb, L.ng, isK && cur.U.psac, L.k_coef, L.k_sigma, r);
+    auto load_ids = [&](const TileCursor& c) -> uint64_t {  // 4 ids | 4 zero bytes << 32
+      uint64_t v = 0;
+      if (c.valid() && c.U.hb) {
+        const uint8_t* tb = c.U.hb + L.tiles_off + (int64_t)c.tl * L.tile_bytes;
+        const int nv = c.nvalid();
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const int row = wrow + 8 * p;
+          if (row < nv)
+            v |= ((uint64_t)tb[o_ids + row] << (8 * p)) | ((uint64_t)tb[o_zeros + (int64_t)row * L.zb] << (32 + 8 * p));
+        }
+      }
+      return v;
+    };
+    uint64_t idn = load_ids(cur);
     uint32_t jt = 0;
     bool ok = true;
     while (cur.valid()) {
-      const RowPack pk = nxt;
+      const uint64_t idc = idn;
       TileCursor nc = cur;
       nc.next(a, S, h);
-      if (nc.valid() && nc.U.hb && row < nc.nvalid())
-        nxt = load_pack(nc.U.hb + L.tiles_off + (int64_t)nc.tl * L.tile_bytes, row, o_codes, o_scales, o_ids,
-                        o_zeros, L.zb, L.ng, isK && nc.U.psac, L.k_coef, L.k_sigma, r);
+      idn = load_ids(nc);
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
-      const bool rvalid = row < cur.nvalid();
+      const int nv = cur.nvalid();
       if (!mbar_wait(bar((isK ? B_KEMPTY : B_VEMPTY) + st), ph ^ 1)) {
         ok = false;
         break;
       }
       uint8_t* dst = sm + (isK ? OFF_K : OFF_V) + st * 2 * BLK;
-      if (!rvalid) {
-        zero_row(dst, row, 0, 16);
-      } else if (!cur.U.hb) {
-        copy_row(dst, row, (isK ? a.kcur : a.vcur) + ((size_t)(cur.tl * 128 + row) * H + h) * 128);
-      } else {
-        dequant_row(dst, row, pk, L.ng, gshift, cur.U.hb + (isK ? L.ktab : L.vtab));
-      }
-      if (isK && cur.U.psac) {
-        uint8_t* sC = sm + OFF_C;
-        const int ch0 = (st * rpad) / 8;
-        if (rvalid) {
-          const float sg = __half2float(__ushort_as_half((unsigned short)pk.sg));
-          const uint32_t cwd[8] = {pk.cf0.x, pk.cf0.y, pk.cf0.z, pk.cf0.w, pk.cf1.x, pk.cf1.y, pk.cf1.z, pk.cf1.w};
+      const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
+      const uint8_t* tab = cur.U.hb ? cur.U.hb + (isK ? L.ktab : L.vtab) : nullptr;
 #pragma unroll
-          for (int c2 = 0; c2 < 4; ++c2) {
-            if (c2 * 8 < rpad) {
-              uint32_t w4[4];
+      for (int rd = 0; rd < 2; ++rd) {
+        uint32_t mv[2][2][8];  // [pass][slice][words]
+        uint32_t cwv[2][2];
+        uint32_t scv[2][2];
 #pragma unroll
-              for (int q2 = 0; q2 < 4; ++q2) {
-                const int j = c2 * 8 + 2 * q2;
-                const uint32_t wd = cwd[j >> 2];
-                const float t0 = j < r ? (float)(int8_t)(wd >> (8 * (j & 3))) * sg : 0.0f;
-                const float t1 = j + 1 < r ? (float)(int8_t)(wd >> (8 * ((j + 1) & 3))) * sg : 0.0f;
-                w4[q2] = pack_f16(t0, t1);
-              }
-              st_chunk(sC, row, ch0 + c2, make_uint4(w4[0], w4[1], w4[2], w4[3]));
+        for (int pp = 0; pp < 2; ++pp) {
+          const int p = 2 * rd + pp;
+          const int row = wrow + 8 * p;
+#pragma unroll
+          for (int sl = 0; sl < 2; ++sl) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mv[pp][sl][e] = 0u;
+            cwv[pp][sl] = 0u;
+            scv[pp][sl] = 0u;
+          }
+          if (row < nv) {
+            if (tb) {
+              const uint8_t* mu = tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256;
+              ldg32B(mu + 32 * q, mv[pp][0]);
+              ldg32B(mu + 128 + 32 * q, mv[pp][1]);
+              const uint8_t* cp = tb + o_codes + row * 32;
+              cwv[pp][0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
+              cwv[pp][1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
+              const unsigned short* sp = reinterpret_cast<const unsigned short*>(tb + o_scales + (int64_t)row * L.ng * 2);
+              scv[pp][0] = __ldg(sp + ((16 * q) >> gshift));
+              scv[pp][1] = __ldg(sp + ((64 + 16 * q) >> gshift));
+            } else {
+              const __nv_bfloat16* src = (isK ? a.kcur : a.vcur) + ((size_t)(cur.tl * 128 + row) * H + h) * 128;
+              const uint4 v0 = ldg16(src + 16 * q), v1 = ldg16(src + 16 * q + 8);
+              const uint4 v2 = ldg16(src + 64 + 16 * q), v3 = ldg16(src + 64 + 16 * q + 8);
+              const uint4 f0 = bf16x8_to_f16x8(v0), f1 = bf16x8_to_f16x8(v1);
+              const uint4 f2 = bf16x8_to_f16x8(v2), f3 = bf16x8_to_f16x8(v3);
+              mv[pp][0][0] = f0.x; mv[pp][0][1] = f0.y; mv[pp][0][2] = f0.z; mv[pp][0][3] = f0.w;
+              mv[pp][0][4] = f1.x; mv[pp][0][5] = f1.y; mv[pp][0][6] = f1.z; mv[pp][0][7] = f1.w;
+              mv[pp][1][0] = f2.x; mv[pp][1][1] = f2.y; mv[pp][1][2] = f2.z; mv[pp][1][3] = f2.w;
+              mv[pp][1][4] = f3.x; mv[pp][1][5] = f3.y; mv[pp][1][6] = f3.z; mv[pp][1][7] = f3.w;
             }
           }
-        } else {
-          zero_row(sC, row, ch0, rpad / 8);
+        }
+#pragma unroll
+        for (int pp = 0; pp < 2; ++pp) {
+          const int p = 2 * rd + pp;
+          const int row = wrow + 8 * p;
+          const uint32_t zbyte = (uint32_t)((idc >> (32 + 8 * p)) & 0xFFu);
+#pragma unroll
+          for (int sl = 0; sl < 2; ++sl) {
+            const int c0 = 8 * sl + 2 * q;  // first of the two chunks of this slice
+            uint32_t ow[8];
+            if (tb && row < nv) {
+              const int g = (64 * sl + 16 * q) >> gshift;
+              const uint32_t sb = scv[pp][sl];
+              const __half2 s2 = u2h(sb | (sb << 16));
+              const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
+              const __half2 z2 = u2h(zz | (zz << 16));
+              const uint32_t word = cwv[pp][sl];
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {  // channel pairs (2k, 2k+1) of the 16-channel word
+                const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+                ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[pp][sl][k])));
+              }
+            } else {
+#pragma unroll
+              for (int k = 0; k < 8; ++k) ow[k] = mv[pp][sl][k];
+            }
+            st_chunk(dst, row, c0, make_uint4(ow[0], ow[1], ow[2], ow[3]));
+            st_chunk(dst, row, c0 + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]));
+          }
+        }
+      }
+      if (isK && cur.U.psac && q * 8 < rpad) {
+        // C_hat = t * sigma, chunk q of the PSAC columns of each of the 4 rows
+        uint8_t* sC = sm + OFF_C;
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const int row = wrow + 8 * p;
+          uint32_t w4[4] = {0u, 0u, 0u, 0u};
+          if (row < nv && q * 8 < r) {
+            const float sg = __half2float(*reinterpret_cast<const __half*>(tb + L.k_sigma + row * 2));
+            const uint2 cw = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)row * r + q * 8));
+            const uint32_t cwd[2] = {cw.x, cw.y};
+#pragma unroll
+            for (int q2 = 0; q2 < 4; ++q2) {
+              const uint32_t wd = cwd[q2 >> 1];
+              w4[q2] = pack_f16((float)(int8_t)(wd >> (16 * (q2 & 1))) * sg, (float)(int8_t)(wd >> (16 * (q2 & 1) + 8)) * sg);
+            }
+          }
+          st_chunk(sC, row, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]));
         }
       }
       fence_proxy_async_smem();
