@@ -15,9 +15,13 @@
  * Eq. 17 compensated logits).
  *
  * Arithmetic: scalar fp32 in a fixed, sequential order for every quantity that
- * decides an integer (centroid ids, INT2 codes, fp16 scales, INT8 PSAC codes);
- * the library must be compiled with -ffp-contract=off so that no multiply-add
- * is fused.  Reconstruction and attention are evaluated in fp64.
+ * decides an integer (centroid ids, INT2 codes, fp16 scales, INT8 PSAC codes).
+ * The sums of products that the paper writes as exact inner products (the
+ * Query-aware distance, the PSAC projection and the two error sums of the
+ * keep rule) take one fused multiply-add (fmaf, a single rounding) per term,
+ * in channel order; every other multiply and add is rounded on its own, so
+ * the library is compiled with -ffp-contract=off and fuses nothing else.
+ * Reconstruction and attention are evaluated in fp64.
  *
  * Readings of the paper where it is silent (rounding, zero-point range, scale
  * storage, INT8 coefficient scheme, keep rule, k-means initialisation) are
@@ -270,7 +274,7 @@ static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uin
  *
  * Per token i and head h:
  *  1. Query-aware distance (Sec. 4.1, Eq. 9): dQ_j = sum_c w_c (k_c - mu_jc)^2,
- *     summed over c in order, each term w_c * (t * t).  w = NULL means w = 1
+ *     summed over c in order, acc = fma(w_c, t * t, acc).  w = NULL means w = 1
  *     (the cold-start rule of App. C.3); Values always use w = 1.
  *  2. Candidates: the M smallest (dQ_j, j) in lexicographic order (ties to the
  *     lower index); M >= C means every centroid (App. C.5).
@@ -281,12 +285,14 @@ static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uin
  *  4. INT2 residual quantization of x = k - mu_id per group of G channels
  *     (Sec. 2, Eq. 1-2, see int2_group) and k0_c = mu_id,c + s (q_c - z).
  *  5. PSAC (Sec. 4.2, Eq. 13 and 16), Keys only, when U is given and r > 0:
- *     E = k - k0; c_j = sum_c E_c U_cj (in order); a = max_j |c_j|;
+ *     E = k - k0; c_j = sum_c E_c U_cj (in order, one fma per term);
+ *     a = max_j |c_j|;
  *     sigma = fp16 round-up of a / 127; t_j = clip(round(c_j * (1/sigma)),
  *     -127, 127) (reading: symmetric absmax INT8, App. D.1 gives INT8 codes
  *     with one FP16 scale per row); chat_j = t_j sigma; e'_c = E_c -
- *     sum_j U_cj chat_j; the row is kept only when sum_c w_c e'_c^2 is
- *     strictly below sum_c w_c E_c^2 (App. D.1: keep a correction only when it
+ *     sum_j U_cj chat_j (fma per term); the row is kept only when
+ *     sum_c w_c e'_c^2 is strictly below sum_c w_c E_c^2 (both fma per term
+ *     on the rounded squares; App. D.1: keep a correction only when it
  *     lowers the approximated Query-weighted error; reading: the diagonal-w
  *     form of Eq. 8); otherwise codes and sigma are zero.
  *
@@ -359,8 +365,7 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
         for (int c = 0; c < d; ++c) {
           float t = k[c] - oracle_bf16_to_f32(mu[c]);
           float t2 = t * t;
-          float wt = wv[c] * t2;
-          acc = acc + wt;
+          acc = fmaf(wv[c], t2, acc); /* one fused multiply-add per term */
         }
         dq[j] = acc;
         chosen[j] = 0;
@@ -463,8 +468,7 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
       for (int j = 0; j < r; ++j) {
         float acc = 0.0f;
         for (int c = 0; c < d; ++c) {
-          float p = E[c] * oracle_bf16_to_f32(Uh[(size_t)c * r + j]);
-          acc = acc + p;
+          acc = fmaf(E[c], oracle_bf16_to_f32(Uh[(size_t)c * r + j]), acc);
         }
         cj[j] = acc;
         float ab = fabsf(acc);
@@ -502,17 +506,12 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
       float errq = 0.0f, err0 = 0.0f;
       for (int c = 0; c < d; ++c) {
         float u = 0.0f;
-        for (int j = 0; j < r; ++j) {
-          float p = oracle_bf16_to_f32(Uh[(size_t)c * r + j]) * chat[j];
-          u = u + p;
-        }
+        for (int j = 0; j < r; ++j) u = fmaf(oracle_bf16_to_f32(Uh[(size_t)c * r + j]), chat[j], u);
         float ep = E[c] - u;
         float e2 = ep * ep;
-        float we = wv[c] * e2;
-        errq = errq + we;
+        errq = fmaf(wv[c], e2, errq);
         float E2 = E[c] * E[c];
-        float wE = wv[c] * E2;
-        err0 = err0 + wE;
+        err0 = fmaf(wv[c], E2, err0);
       }
       int keep = errq < err0;
       float gk = rel_gap(errq, err0);
