@@ -1,24 +1,47 @@
-// append.cu -- quantize-on-append with a tensor-core distance filter.
+// append.cu -- quantize-on-append: a tensor-core candidate filter followed by
+// the exact per-token quantisation.
 //
-// Per CTA: 128 new tokens of one head, Keys (blockIdx.z = 0) or Values (1);
-// thread = token.  Steps (Sec. 4.1 QSAC, Sec. 2 Eq. 1-4 INT2, Sec. 4.2 PSAC):
-//   1. Candidate filter on tcgen05: D = K (w o mu)^T for all C centroids in
-//      one f16 MMA into TMEM, so that dQ_j - sum_c w_c k_c^2 = A_j - 2 D_j
-//      with A_j = sum_c w_c mu_jc^2 (Eq. 9 expanded).  The f16 rounding of
-//      w o mu and the fp32 accumulation give an error below
-//      B = 2^-9 |k| max_j |w o mu_j| + 2^-15 max_j A_j + 2^-18 (|k| + ...)
-//      (a bound with a 4x margin over the f16 rounding term), so every
-//      centroid among the true top-M lies within 2B of the M-th smallest
-//      filtered distance.  When exactly M centroids fall inside that band
-//      they are the top-M; otherwise the band members are rescored with the
-//      exact Query-aware distance (fp32, channel order) and the M smallest
-//      (ties to the lower index) kept.
-//   2. QSAC score (Eq. 10, 12) of each candidate, INT2 residual quantisation
-//      and packing, and for Keys the PSAC coefficients with the keep rule, all
-//      with explicitly rounded fp32 operations in channel order, identical to
-//      a sequential evaluation of the formulas.
+// Kernel 1, append_filter (persistent, one CTA per SM, two groups of 128
+// token rows).  For a run of 128-token tiles of one (head, K/V side):
+//   * once per run, B = w o mu for all C centroids (Sec. 4.1, Eq. 9 expanded
+//     as dQ_j = sum_c w_c k_c^2 - 2 D_j + A_j with D = K (w o mu)^T and
+//     A_j = sum_c w_c mu_jc^2) is split into two binary16 operands
+//     B_hi = f16(w o mu), B_lo = f16(w o mu - B_hi), so that B_hi + B_lo
+//     carries w o mu to 2^-22 relative;
+//   * per tile, the bf16 token rows arrive by TMA (128-byte swizzled), are
+//     converted in place to binary16, and two tcgen05 MMAs accumulate
+//     D = K B_hi^T + K B_lo^T (fp32, 128 x C) in TMEM;
+//   * each thread reads its row of D and keeps the M+1 smallest
+//     dt_j = A_j - 2 D_j.  With the error bound B of dt (the split operand,
+//     the fp32 accumulation, and the fp32 rounding of the sequential
+//     Query-aware distance the selection is defined on), every centroid of
+//     the exact top-M lies within 2B of the M-th smallest dt; when the
+//     (M+1)-th lies beyond that band the top-M is decided, otherwise the band
+//     members (at most 16) are listed for exact rescoring.
+//   The decision record of a token (count byte + up to 16 centroid ids) is
+//   parked in the token's own 32 code bytes of the destination slot.
+//
+// Kernel 2, append_quant (one CTA per 128-token tile, thread = token; the
+// tile arrives by TMA).  It reads the record, rescores band members exactly
+// when needed, evaluates the QSAC score (Eq. 10, 12) of each candidate, and
+// quantises the residual to INT2 (Eq. 1-2) with packing.  For Keys, the same
+// channel pass accumulates the PSAC projection c = U_r^T E (Eq. 13) in
+// channel order (one fused multiply-add per term) together with
+// v = U_r^T (w o E) and err0 = sum_c w_c E_c^2;
+// the keep rule (Eq. 16, diagonal-w form) compares
+// errq - err0 = chat^T (U^T W U) chat - 2 chat.v against a rigorous bound of
+// its difference to the sequential evaluation, and evaluates the two sums
+// sequentially only when they are too close to call.  All arithmetic that
+// decides an output is fp32 in channel order with every rounding explicit:
+// a separately rounded multiply or add, or one fused multiply-add per term
+// of a sum of products (packed two lanes at a time where the lanes are
+// independent), identical to the sequential evaluation of the formulas.
+//
 // M >= C skips the filter (every centroid is a candidate); 8 < M < C goes to
 // the generic kernel (append_generic.cu).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
 
@@ -27,66 +50,26 @@ namespace {
 
 using namespace ptx;
 
-constexpr int NT = 128;        // threads = tokens per CTA
 constexpr int kMaxFilterM = 8;
-constexpr int kBand = 16;      // band members rescored exactly before falling back to all C
+constexpr int kBand = 16;         // band members listed for exact rescoring
+constexpr int kRecAll = 255;      // record: rescore every centroid
 
-constexpr int OFF_A = 0;                          // K tile, f16, 2 blocks of 128 x 128 B
-constexpr int OFF_B = 32768;                      // w o mu, f16, 2 blocks of Npad x 128 B
-constexpr int OFF_AJ = OFF_B + 65536;             // A_j [256] fp32
-constexpr int OFF_W = OFF_AJ + 1024;              // w [128]
-constexpr int OFF_WG = OFF_W + 512;               // W_g [4]
-constexpr int OFF_RED = OFF_WG + 16;              // [4 warps][2] maxima
-constexpr int OFF_U = OFF_RED + 48;               // U [128][r] bf16 (<= 8 KB)
-constexpr int OFF_LIST = OFF_U + 8192;            // band lists [128][16] u8
-constexpr int OFF_BAR = OFF_LIST + NT * kBand;    // mbarrier + TMEM slot
-constexpr int SMEM_BYTES = OFF_BAR + 64 + 1024;   // + alignment slack
-
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+__device__ __forceinline__ uint4 lds16(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
 
-// Swizzled 16-byte store into K-major operand blocks of `rows` rows.
-__device__ __forceinline__ void st_chunk_rows(uint8_t* base, int rows, int row, int ch, uint4 v) {
-  const int kb = ch >> 3, pos = (ch & 7) ^ (row & 7);
-  *reinterpret_cast<uint4*>(base + (size_t)kb * rows * 128 + row * 128 + pos * 16) = v;
-}
-
-__device__ __forceinline__ void unpack8(const uint4 v, float (&f)[8]) {
-  f[0] = bf_lo(v.x); f[1] = bf_hi(v.x); f[2] = bf_lo(v.y); f[3] = bf_hi(v.y);
-  f[4] = bf_lo(v.z); f[5] = bf_hi(v.z); f[6] = bf_lo(v.w); f[7] = bf_hi(v.w);
-}
-__device__ __forceinline__ float sel4(const float (&a)[4], int g) {
-  return g == 0 ? a[0] : (g == 1 ? a[1] : (g == 2 ? a[2] : a[3]));
-}
-__device__ __forceinline__ int sel4i(const int (&a)[4], int g) {
-  return g == 0 ? a[0] : (g == 1 ? a[1] : (g == 2 ? a[2] : a[3]));
+// Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in a
+// pair of 128-byte-swizzled blocks of `rows` rows x 64 two-byte elements.
+__device__ __forceinline__ int sw_off(int rows, int row, int ch) {
+  return (ch >> 3) * rows * 128 + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
 }
 
-// Exact Query-aware distance (Eq. 9) in channel order: xr is the token row,
-// mu the centroid row (bf16), sW the weights.
-__device__ __forceinline__ float exact_dq(const __nv_bfloat16* xr, const __nv_bfloat16* mu, const float* sW) {
-  float acc = 0.0f;
-#pragma unroll 1
-  for (int ch = 0; ch < 16; ++ch) {
-    float kf[8], mf[8];
-    unpack8(ldg16(xr + ch * 8), kf);
-    unpack8(ldg16(mu + ch * 8), mf);
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const float t = __fsub_rn(kf[e], mf[e]);
-      acc = __fadd_rn(acc, __fmul_rn(sW[ch * 8 + e], __fmul_rn(t, t)));
-    }
-  }
-  return acc;
-}
-
-// Insert (v, j) into the ascending list of the Mc smallest (value, index)
+// Insert (v, j) into the ascending list of the n smallest (value, index)
 // pairs; indices arrive in ascending order, so an equal value stays behind.
-__device__ __forceinline__ void insert_top(float (&tv)[kMaxFilterM], int (&tj)[kMaxFilterM], int Mc, float v, int j) {
+template <int CAP>
+__device__ __forceinline__ void insert_top(float (&tv)[CAP], int (&tj)[CAP], int n, float v, int j) {
 #pragma unroll
-  for (int s = 0; s < kMaxFilterM; ++s) {
-    if (s < Mc && v < tv[s]) {
+  for (int s = 0; s < CAP; ++s) {
+    if (s < n && v < tv[s]) {
       const float ov = tv[s];
       const int oj = tj[s];
       tv[s] = v;
@@ -96,458 +79,848 @@ __device__ __forceinline__ void insert_top(float (&tv)[kMaxFilterM], int (&tj)[k
     }
   }
 }
-__device__ __forceinline__ float kth_of(const float (&tv)[kMaxFilterM], int Mc) {
+template <int CAP>
+__device__ __forceinline__ float sel_at(const float (&tv)[CAP], int i) {
   float k = tv[0];
 #pragma unroll
-  for (int s = 1; s < kMaxFilterM; ++s)
-    if (s == Mc - 1) k = tv[s];
+  for (int s = 1; s < CAP; ++s)
+    if (s == i) k = tv[s];
   return k;
 }
 
-template <int R, int GS>
-__global__ void __launch_bounds__(NT, 2) append_kernel(const AppendArgs a) {
+// ============================================================================
+// Kernel 1: candidate filter
+// ============================================================================
+constexpr int FG = 2;                       // token groups per CTA
+constexpr int FNT = FG * 128;
+constexpr int F_BHI = 0;                    // [2][256 rows][128 B] f16
+constexpr int F_BLO = 65536;
+constexpr int F_A = 131072;                 // FG x [2][128 rows][128 B]
+constexpr int F_AJ = F_A + FG * 32768;      // A_j [256] fp32
+constexpr int F_W = F_AJ + 1024;            // w [128]
+constexpr int F_RED = F_W + 512;            // [8 warps][2]
+constexpr int F_LIST = F_RED + 64;          // FNT x 32-byte records
+constexpr int F_BAR = F_LIST + FNT * 32;    // 4 mbarriers, flags, TMEM slot
+constexpr int F_SMEM = F_BAR + 64 + 1024;
+
+__global__ void __launch_bounds__(FNT, 1)
+    append_filter(const AppendArgs a, const __grid_constant__ CUtensorMap tm_k,
+                  const __grid_constant__ CUtensorMap tm_v, int tiles, int units) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const Layout& L = a.L;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int h = blockIdx.y;
-  const bool is_key = blockIdx.z == 0;
-  const int64_t t = (int64_t)blockIdx.x * NT + tid;
-  const bool valid = t < a.N;
-  const int C = L.C, H = L.H;
-  constexpr int r = R, G = GS, ng = 128 / GS;
-  const int Mc = a.M;
-  const bool all_cand = Mc >= C;
+  const int g = tid >> 7, row = tid & 127;
+  const int C = L.C, H = L.H, Mc = a.M;
   const int Npad = (C + 15) & ~15;
-  const __nv_bfloat16* x = is_key ? a.k : a.v;
-  const __nv_bfloat16* tab = (is_key ? a.kc : a.vc) + (size_t)h * C * 128;
-  const bool use_w = is_key && a.w != nullptr;
-  const bool psac = is_key && a.U != nullptr && r > 0;
-  uint8_t* head = a.base + head_offset(L, a.slot, h);
 
-  float* sAj = reinterpret_cast<float*>(sm + OFF_AJ);
-  float* sW = reinterpret_cast<float*>(sm + OFF_W);
-  float* sWg = reinterpret_cast<float*>(sm + OFF_WG);
-  float* sRed = reinterpret_cast<float*>(sm + OFF_RED);
-  __nv_bfloat16* sU = reinterpret_cast<__nv_bfloat16*>(sm + OFF_U);
-  uint8_t* myl = sm + OFF_LIST + tid * kBand;
-  const uint32_t bar = smem_u32(sm + OFF_BAR);
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + OFF_BAR + 16);
+  float* sAj = reinterpret_cast<float*>(sm + F_AJ);
+  float* sW = reinterpret_cast<float*>(sm + F_W);
+  float* sRed = reinterpret_cast<float*>(sm + F_RED);
+  uint8_t* myl = sm + F_LIST + tid * 32;
+  const uint32_t bar_tma = smem_u32(sm + F_BAR + 8 * g);
+  const uint32_t bar_mma = smem_u32(sm + F_BAR + 16 + 8 * g);
+  volatile int* flagA = reinterpret_cast<volatile int*>(sm + F_BAR + 32);  // [FG] copy timed out
+  volatile int* flagB = reinterpret_cast<volatile int*>(sm + F_BAR + 40);  // [FG] MMA timed out
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + F_BAR + 48);
+  uint8_t* sA = sm + F_A + g * 32768;
 
-  // The chunk's own tables travel with the slot (one CTA per head and K/V),
-  // stored as binary16 (exact for bf16 values in the binary16 range), the
-  // operand type of the attention kernel's tensor-core path.
-  if (blockIdx.x == 0) {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
-    __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
-    for (int i = tid; i < C * 64; i += NT) {
-      const uint32_t pr = src[i];
-      dst[i] = __floats2half2_rn(bf_lo(pr), bf_hi(pr));
-    }
-    if (psac) {
-      __nv_bfloat16* ut = reinterpret_cast<__nv_bfloat16*>(head + L.ut);
-      const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * r;
-      for (int i = tid; i < r * 128; i += NT) ut[i] = Uh[(size_t)(i % 128) * r + i / 128];  // U_r^T [r][d]
-    }
-  }
-
-  if (!all_cand && warp == 0) {
-    tmem_alloc(smem_u32(tslot), 256);
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tslot), 512);
     tmem_relinquish();
   }
   if (tid == 0) {
-    mbar_init(bar, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(sm + F_BAR + 8 * i), 1);
     fence_mbar_init();
+    flagA[0] = flagA[1] = 0;
+    flagB[0] = flagB[1] = 0;
   }
-  sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
-  if (psac)
-    for (int i = tid; i < 128 * r; i += NT) sU[i] = a.U[(size_t)h * 128 * r + i];  // [d][r]
+  tc_fence_before();
   __syncthreads();
-  if (tid < ng) {
-    float Wg = 0.0f;
-    for (int c = tid * G; c < (tid + 1) * G; ++c) Wg = __fadd_rn(Wg, sW[c]);
-    sWg[tid] = Wg;
-  }
+  tc_fence_after();
+  const uint32_t tbase = *tslot;
+  const uint32_t tD = tbase + (uint32_t)(g * 256);
+  const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
 
-  // ---- this thread's f16 operand row and |k|^2
-  const __nv_bfloat16* xr = x + ((size_t)(valid ? t : 0) * H + h) * 128;
-  float knorm2 = 0.0f;
-  if (!all_cand) {
-#pragma unroll 4
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 v = valid ? ldg16(xr + ch * 8) : make_uint4(0, 0, 0, 0);
-      st_chunk_rows(sm + OFF_A, 128, tid, ch, bf16x8_to_f16x8(v));
-      float kf[8];
-      unpack8(v, kf);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) knorm2 = fmaf(kf[e], kf[e], knorm2);
-    }
-  }
+  const int nb = gridDim.x;
+  const int u0 = (int)((int64_t)blockIdx.x * units / nb);
+  const int u1 = (int)((int64_t)(blockIdx.x + 1) * units / nb);
+  uint32_t ph_tma = 0, ph_mma = 0;
 
-  uint32_t tD = 0;
-  float bandB = 0.0f;
-  if (!all_cand) {
-    // ---- w o mu rows (f16 operand B), A_j and the norms for the bound
-    float wmax2 = 0.0f, amax = 0.0f;
-    for (int j = tid; j < Npad; j += NT) {
-      float A = 0.0f, n2 = 0.0f;
+  for (int s0 = u0; s0 < u1;) {
+    const int pair = s0 / tiles;                 // side * H + h
+    const int s1 = min(u1, (pair + 1) * tiles);
+    const bool is_key = pair < H;
+    const int h = pair % H;
+    const bool use_w = is_key && a.w != nullptr;
+    const __nv_bfloat16* tab = (is_key ? a.kc : a.vc) + (size_t)h * C * 128;
+    const CUtensorMap* tm = is_key ? &tm_k : &tm_v;
+    uint8_t* head = a.base + head_offset(L, a.slot, h);
+    const int64_t o_rec = is_key ? L.k_codes : L.v_codes;
+
+    // ---- B_hi, B_lo and A_j of this (head, side)
+    if (tid < 128) sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
+    __syncthreads();
+    float n2 = 0.0f, amax = 0.0f;
+    {
+      const int j = tid;
       if (j < C) {
         const __nv_bfloat16* mr = tab + (size_t)j * 128;
+        float A = 0.0f;
 #pragma unroll 4
         for (int ch = 0; ch < 16; ++ch) {
           const uint4 m = ldg16(mr + ch * 8);
           const uint32_t mw[4] = {m.x, m.y, m.z, m.w};
-          uint32_t ow[4];
+          uint32_t hw[4], lw[4];
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
-            const float m0 = bf_lo(mw[p]), m1 = bf_hi(mw[p]);
+            const float m0 = __uint_as_float(mw[p] << 16), m1 = __uint_as_float(mw[p] & 0xFFFF0000u);
             const float w0 = __fmul_rn(sW[ch * 8 + 2 * p], m0), w1 = __fmul_rn(sW[ch * 8 + 2 * p + 1], m1);
             A = fmaf(w0, m0, fmaf(w1, m1, A));
             n2 = fmaf(w0, w0, fmaf(w1, w1, n2));
-            ow[p] = pack_f16(w0, w1);
+            const __half2 hh = __floats2half2_rn(w0, w1);
+            const float2 hf = __half22float2(hh);
+            hw[p] = *reinterpret_cast<const uint32_t*>(&hh);
+            lw[p] = pack_f16(w0 - hf.x, w1 - hf.y);
           }
-          st_chunk_rows(sm + OFF_B, Npad, j, ch, make_uint4(ow[0], ow[1], ow[2], ow[3]));
+          const int off = sw_off(Npad, j, ch);
+          *reinterpret_cast<uint4*>(sm + F_BHI + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+          *reinterpret_cast<uint4*>(sm + F_BLO + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
         }
         sAj[j] = A;
+        amax = fabsf(A);
       } else {
+        if (j < Npad) {
 #pragma unroll
-        for (int ch = 0; ch < 16; ++ch) st_chunk_rows(sm + OFF_B, Npad, j, ch, make_uint4(0, 0, 0, 0));
-        sAj[j] = INFINITY;
+          for (int ch = 0; ch < 16; ++ch) {
+            const int off = sw_off(Npad, j, ch);
+            *reinterpret_cast<uint4*>(sm + F_BHI + off) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(sm + F_BLO + off) = make_uint4(0, 0, 0, 0);
+          }
+        }
+        sAj[j] = INFINITY;  // j in [C, 256): never selected
       }
-      wmax2 = fmaxf(wmax2, n2);
-      amax = fmaxf(amax, fabsf(A));
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) {
-      wmax2 = fmaxf(wmax2, __shfl_xor_sync(0xFFFFFFFFu, wmax2, off));
+      n2 = fmaxf(n2, __shfl_xor_sync(0xFFFFFFFFu, n2, off));
       amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, off));
     }
     if (lane == 0) {
-      sRed[2 * warp] = wmax2;
+      sRed[2 * warp] = n2;
       sRed[2 * warp + 1] = amax;
     }
     fence_proxy_async_smem();
-    tc_fence_before();
     __syncthreads();
-    tc_fence_after();
-    tD = *tslot;
-    if (tid == 0) {
-      const uint32_t aA = smem_u32(sm + OFF_A), aB = smem_u32(sm + OFF_B);
-      const uint32_t id = idesc_f16(128, Npad, false);
-#pragma unroll
-      for (int kb = 0; kb < 2; ++kb)
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks)
-          umma_ss(tD, desc_sw128(aA + kb * 16384 + ks * 32), desc_sw128(aB + kb * Npad * 128 + ks * 32), id,
-                  (kb | ks) != 0);
-      umma_commit(bar);
-    }
     float W2 = 0.0f, Am = 0.0f;
 #pragma unroll
-    for (int i = 0; i < NT / 32; ++i) {
+    for (int i = 0; i < FNT / 32; ++i) {
       W2 = fmaxf(W2, sRed[2 * i]);
       Am = fmaxf(Am, sRed[2 * i + 1]);
     }
-    const float kn = sqrtf(knorm2), Wn = sqrtf(W2);
-    bandB = ldexpf(kn * Wn, -9) + ldexpf(Am, -15) + ldexpf(kn + Wn + 1.0f, -18);
-  }
+    const float Wn = sqrtf(W2);
 
-  // ---- 1. candidates
-  int ncand = 0;  // candidates in myl (all_cand: every centroid)
-  bool timeout = false;
-  if (!all_cand) {
-    const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar, 0));
-    if (!ok) {
-      timeout = true;
-    } else {
-      tc_fence_after();
-      const uint32_t lrow = (uint32_t)(warp * 32) << 16;
-      float tv[kMaxFilterM];
-      int tj[kMaxFilterM];
-#pragma unroll
-      for (int s = 0; s < kMaxFilterM; ++s) { tv[s] = INFINITY; tj[s] = 0x7FFFFFFF; }
-      float kth = INFINITY;
-      float v[32];
-      for (int cb = 0; cb * 32 < Npad; ++cb) {
-        tmem_ld32(tD + lrow + cb * 32, v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int j = cb * 32 + e;
-          if (j < C) {
-            const float dt = fmaf(-2.0f, v[e], sAj[j]);
-            if (dt < kth) {
-              insert_top(tv, tj, Mc, dt, j);
-              kth = kth_of(tv, Mc);
-            }
-          }
-        }
+    // ---- the tiles of this run, alternating between the two groups
+    for (int u = s0 + g; u < s1; u += FG) {
+      const int tile = u - pair * tiles;
+      if (row == 0) {
+        mbar_arrive_expect_tx(bar_tma, 32768);
+        tma_load_3d(smem_u32(sA), tm, 0, h, tile * 128, bar_tma);
+        tma_load_3d(smem_u32(sA + 16384), tm, 64, h, tile * 128, bar_tma);
       }
-      const float thr = kth + 2.0f * bandB;
-      int nb = 0;
-      for (int cb = 0; cb * 32 < Npad; ++cb) {
-        tmem_ld32(tD + lrow + cb * 32, v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int j = cb * 32 + e;
-          if (j < C && fmaf(-2.0f, v[e], sAj[j]) <= thr) {
-            if (nb < kBand) myl[nb] = (uint8_t)j;
-            ++nb;
-          }
-        }
-      }
-      if (valid) {
-        if (nb == Mc) {
-          ncand = Mc;
-        } else {
-          // rescore exactly: the band members, or every centroid if the band overflowed
-          float ev[kMaxFilterM];
-          int ej[kMaxFilterM];
-#pragma unroll
-          for (int s = 0; s < kMaxFilterM; ++s) { ev[s] = INFINITY; ej[s] = 0x7FFFFFFF; }
-          float ek = INFINITY;
-          const int n_eval = nb <= kBand ? nb : C;
-          for (int m = 0; m < n_eval; ++m) {
-            const int j = nb <= kBand ? myl[m] : m;
-            const float dq = exact_dq(xr, tab + (size_t)j * 128, sW);
-            if (dq < ek) {
-              insert_top(ev, ej, Mc, dq, j);
-              ek = kth_of(ev, Mc);
-            }
-          }
-#pragma unroll
-          for (int s = 0; s < kMaxFilterM; ++s)
-            if (s < Mc) myl[s] = (uint8_t)ej[s];
-          ncand = Mc;
-        }
-      }
-    }
-  } else {
-    ncand = C;
-  }
+      if (!mbar_wait(bar_tma, ph_tma)) flagA[g] = 1;
+      ph_tma ^= 1;
 
-  // ---- 2. QSAC score over the candidates (Eq. 10, 12), lowest (S, j)
-  if (valid && !timeout) {
-    float bestS = INFINITY;
-    int bestj = 0x7FFFFFFF;
-    for (int m = 0; m < ncand; ++m) {
-      const int j = all_cand ? m : myl[m];
-      const __nv_bfloat16* mr = tab + (size_t)j * 128;
-      float mx[4], mn[4];
-#pragma unroll
-      for (int g = 0; g < 4; ++g) { mx[g] = -INFINITY; mn[g] = INFINITY; }
-#pragma unroll
+      // bf16 row -> binary16 in place; |k|^2, sum_c w_c k_c^2, max |k_c|
+      float kn2 = 0.0f, K0 = 0.0f, kmx = 0.0f;
+#pragma unroll 4
       for (int ch = 0; ch < 16; ++ch) {
-        float kf[8], mf[8];
-        unpack8(ldg16(xr + ch * 8), kf);
-        unpack8(ldg16(mr + ch * 8), mf);
-        const int g = (ch * 8) / G;
+        uint4* p = reinterpret_cast<uint4*>(sA + sw_off(128, row, ch));
+        const uint4 v = *p;
+        const uint32_t vw[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float rc = __fsub_rn(kf[e], mf[e]);
-          mx[g] = fmaxf(mx[g], rc);
-          mn[g] = fminf(mn[g], rc);
+        for (int q = 0; q < 4; ++q) {
+          const float k0 = __uint_as_float(vw[q] << 16), k1 = __uint_as_float(vw[q] & 0xFFFF0000u);
+          kn2 = fmaf(k0, k0, fmaf(k1, k1, kn2));
+          K0 = fmaf(sW[ch * 8 + 2 * q] * k0, k0, fmaf(sW[ch * 8 + 2 * q + 1] * k1, k1, K0));
+          kmx = fmax3f(kmx, fabsf(k0), fabsf(k1));
         }
+        *p = bf16x8_to_f16x8(v);
       }
-      float S = 0.0f;
-#pragma unroll
-      for (int g = 0; g < 4; ++g) {
-        if (g < ng) {
-          const float Rg = __fsub_rn(mx[g], mn[g]);
-          S = __fadd_rn(S, __fmul_rn(sWg[g], __fmul_rn(Rg, Rg)));
-        }
-      }
-      if (S < bestS || (S == bestS && j < bestj)) { bestS = S; bestj = j; }
-    }
-    const int id = bestj < C ? bestj : C - 1;
-    const __nv_bfloat16* mr = tab + (size_t)id * 128;
-
-    // ---- 3. INT2 residual quantisation (Eq. 1-2) of x = k - mu_id
-    float lo[4], hi[4];
-#pragma unroll
-    for (int g = 0; g < 4; ++g) { lo[g] = 0.0f; hi[g] = 0.0f; }
-#pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      float kf[8], mf[8];
-      unpack8(ldg16(xr + ch * 8), kf);
-      unpack8(ldg16(mr + ch * 8), mf);
-      const int g = (ch * 8) / G;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const float xc = __fsub_rn(kf[e], mf[e]);
-        lo[g] = fminf(lo[g], xc);
-        hi[g] = fmaxf(hi[g], xc);
-      }
-    }
-    float sc[4], inv[4];
-    int zq[4];
-    __half sh[4];
-    uint32_t zbyte = 0;
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      sc[g] = 0.0f; inv[g] = 0.0f; zq[g] = 0; sh[g] = __ushort_as_half(0);
-      if (g < ng) {
-        sh[g] = __float2half_ru(__fdiv_rn(__fsub_rn(hi[g], lo[g]), 3.0f));
-        sc[g] = __half2float(sh[g]);
-        if (sc[g] != 0.0f) {
-          inv[g] = __frcp_rn(sc[g]);
-          const int z = (int)rintf(__fmul_rn(-lo[g], inv[g]));
-          zq[g] = z < 0 ? 0 : (z > 3 ? 3 : z);
-        }
-        zbyte |= (uint32_t)zq[g] << (2 * g);
-      }
-    }
-    const int64_t tile = t / kTile;
-    const int rowi = (int)(t % kTile);
-    uint8_t* tb = head + L.tiles_off + tile * L.tile_bytes;
-    uint32_t* dcodes = reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_codes : L.v_codes) + rowi * 32);
-    // 16 channels per word: even channel 2k at bits 2k, odd channel 2k+1 at 16 + 2k
-#pragma unroll 1
-    for (int wd = 0; wd < 8; ++wd) {
-      uint32_t word = 0;
-#pragma unroll
-      for (int hc = 0; hc < 2; ++hc) {
-        const int ch = 2 * wd + hc;
-        float kf[8], mf[8];
-        unpack8(ldg16(xr + ch * 8), kf);
-        unpack8(ldg16(mr + ch * 8), mf);
-        const int g = (ch * 8) / G;
-        const float s = sel4(sc, g), iv = sel4(inv, g);
-        const int z = sel4i(zq, g);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float xc = __fsub_rn(kf[e], mf[e]);
-          int q = 0;
-          if (s != 0.0f) {
-            q = (int)rintf(__fmul_rn(xc, iv)) + z;
-            q = q < 0 ? 0 : (q > 3 ? 3 : q);
-          }
-          const int j16 = 8 * hc + e;
-          word |= (uint32_t)q << (16 * (j16 & 1) + 2 * (j16 >> 1));
-        }
-      }
-      dcodes[wd] = word;
-    }
-    __half* dsc = reinterpret_cast<__half*>(tb + (is_key ? L.k_scales : L.v_scales) + (int64_t)rowi * ng * 2);
-#pragma unroll
-    for (int g = 0; g < 4; ++g)
-      if (g < ng) dsc[g] = sh[g];
-    tb[(is_key ? L.k_ids : L.v_ids) + rowi] = (uint8_t)id;
-    uint8_t* dz = tb + (is_key ? L.k_zeros : L.v_zeros) + (int64_t)rowi * L.zb;
-    dz[0] = (uint8_t)zbyte;
-    for (int b = 1; b < L.zb; ++b) dz[b] = 0;
-
-    // ---- 4. PSAC (Eq. 13, 16) with the keep rule, Keys only
-    if constexpr (R > 0) {
-      if (is_key) {
-        int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)rowi * R);
-        __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma) + rowi;
-        if (!psac) {
-#pragma unroll
-          for (int j = 0; j < R; ++j) coef[j] = 0;
-          *sig = __ushort_as_half(0);
-        } else {
-          // E_c = k_c - k0_c, k0_c = mu_c + s (q_c - z); q_c re-read from the packed word
-          float cj[R];
-#pragma unroll
-          for (int j = 0; j < R; ++j) cj[j] = 0.0f;
-#pragma unroll 1
-          for (int ch = 0; ch < 16; ++ch) {
-            float kf[8], mf[8];
-            unpack8(ldg16(xr + ch * 8), kf);
-            unpack8(ldg16(mr + ch * 8), mf);
-            const int g = (ch * 8) / G;
-            const float s = sel4(sc, g);
-            const int z = sel4i(zq, g);
-            const uint32_t word = dcodes[ch >> 1];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const int j16 = 8 * (ch & 1) + e;
-              const int q = (word >> (16 * (j16 & 1) + 2 * (j16 >> 1))) & 3;
-              const float E = __fsub_rn(kf[e], __fadd_rn(mf[e], __fmul_rn((float)(q - z), s)));
-              const __nv_bfloat16* ur = sU + (ch * 8 + e) * R;
-#pragma unroll
-              for (int j = 0; j < R; ++j) cj[j] = __fadd_rn(cj[j], __fmul_rn(E, __bfloat162float(ur[j])));
-            }
-          }
-          float amax = 0.0f;
-#pragma unroll
-          for (int j = 0; j < R; ++j) amax = fmaxf(amax, fabsf(cj[j]));
-          const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
-          const float sg = __half2float(sgh);
-          const float sinv = sg != 0.0f ? __frcp_rn(sg) : 0.0f;
-#pragma unroll
-          for (int j = 0; j < R; ++j) {  // cj becomes chat = t * sigma
-            const float qq = sg != 0.0f ? fminf(fmaxf(rintf(__fmul_rn(cj[j], sinv)), -127.0f), 127.0f) : 0.0f;
-            cj[j] = __fmul_rn(qq, sg);
-          }
-          // keep only if sum_c w_c (E_c - (U chat)_c)^2 < sum_c w_c E_c^2, both in channel order
-          float errq = 0.0f, err0 = 0.0f;
-#pragma unroll 1
-          for (int ch = 0; ch < 16; ++ch) {
-            float kf[8], mf[8];
-            unpack8(ldg16(xr + ch * 8), kf);
-            unpack8(ldg16(mr + ch * 8), mf);
-            const int g = (ch * 8) / G;
-            const float s = sel4(sc, g);
-            const int z = sel4i(zq, g);
-            const uint32_t word = dcodes[ch >> 1];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const int c = ch * 8 + e;
-              const int j16 = 8 * (ch & 1) + e;
-              const int q = (word >> (16 * (j16 & 1) + 2 * (j16 >> 1))) & 3;
-              const float E = __fsub_rn(kf[e], __fadd_rn(mf[e], __fmul_rn((float)(q - z), s)));
-              const __nv_bfloat16* ur = sU + c * R;
-              float u = 0.0f;
-#pragma unroll
-              for (int j = 0; j < R; ++j) u = __fadd_rn(u, __fmul_rn(__bfloat162float(ur[j]), cj[j]));
-              const float ep = __fsub_rn(E, u);
-              errq = __fadd_rn(errq, __fmul_rn(sW[c], __fmul_rn(ep, ep)));
-              err0 = __fadd_rn(err0, __fmul_rn(sW[c], __fmul_rn(E, E)));
-            }
-          }
-          const bool keep = errq < err0;
-#pragma unroll
-          for (int j = 0; j < R; ++j) coef[j] = keep ? (int8_t)(int)rintf(__fmul_rn(cj[j], sinv)) : (int8_t)0;
-          *sig = keep ? sgh : __ushort_as_half(0);
-        }
-      }
-    }
-  }
-  if (timeout && tid == 0) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_TIMEOUT);
-
-  if (!all_cand) {
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) {
+      fence_proxy_async_smem();
+      tc_fence_before();
+      named_bar_sync(1 + g, 128);
       tc_fence_after();
-      tmem_dealloc(tD, 256);
+      if (flagA[g]) break;
+      if (row == 0) {
+        const uint32_t aA = smem_u32(sA);
+        const uint32_t id = idesc_f16(128, Npad, false);
+#pragma unroll
+        for (int hl = 0; hl < 2; ++hl) {
+          const uint32_t aB = smem_u32(sm + (hl ? F_BLO : F_BHI));
+#pragma unroll
+          for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+              umma_ss(tD, desc_sw128(aA + kb * 16384 + ks * 32), desc_sw128(aB + kb * Npad * 128 + ks * 32), id,
+                      (hl | kb | ks) != 0);
+        }
+        umma_commit(bar_mma);
+      }
+      if (!mbar_wait(bar_mma, ph_mma)) flagB[g] = 1;
+      ph_mma ^= 1;
+      tc_fence_after();
+
+      // ---- M+1 smallest dt_j of this row
+      constexpr int CAP = kMaxFilterM + 1;
+      float tv[CAP];
+      int tj[CAP];
+#pragma unroll
+      for (int s = 0; s < CAP; ++s) { tv[s] = INFINITY; tj[s] = 0x7FFFFFFF; }
+      float thr = INFINITY;  // the (M+1)-th smallest so far
+      for (int cb = 0; cb * 32 < Npad; ++cb) {
+        float v[32];
+        __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the insertions
+        tmem_ld32(tD + lrow + cb * 32, v);
+        const float4* aj4 = reinterpret_cast<const float4*>(sAj + cb * 32);
+#pragma unroll
+        for (int e = 0; e < 32; e += 4) {
+          const float4 A4 = aj4[e >> 2];
+          v[e] = fmaf(-2.0f, v[e], A4.x);
+          v[e + 1] = fmaf(-2.0f, v[e + 1], A4.y);
+          v[e + 2] = fmaf(-2.0f, v[e + 2], A4.z);
+          v[e + 3] = fmaf(-2.0f, v[e + 3], A4.w);
+        }
+        float mn = fmin3(v[0], v[1], v[2]);
+#pragma unroll
+        for (int e = 3; e < 31; e += 2) mn = fmin3(mn, v[e], v[e + 1]);
+        mn = fminf(mn, v[31]);
+        if (mn < thr) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            if (v[e] < thr) {
+              insert_top(tv, tj, Mc + 1, v[e], cb * 32 + e);
+              thr = sel_at(tv, Mc);
+            }
+          }
+        }
+      }
+      const float kth = sel_at(tv, Mc - 1);
+      const float kn = sqrtf(kn2);
+      const float Bb = ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
+      const float lim = kth + 2.0f * Bb;
+      const bool over = !(kmx <= 65504.0f) || !(kn2 < INFINITY) || !(lim < INFINITY);
+      const bool decided = !over && thr > lim;
+      int n = over ? kRecAll : Mc;
+      if (decided) {
+#pragma unroll
+        for (int s = 0; s < kMaxFilterM; ++s)
+          if (s < Mc) myl[1 + s] = (uint8_t)tj[s];
+      }
+      // The band (every j with dt_j <= kth + 2B, ascending j) of the rows
+      // that are not decided; the TMEM reads are warp-collective, so the
+      // whole warp walks the row blocks whenever one of its rows needs it.
+      const bool need_band = !over && !decided;
+      if (__any_sync(0xFFFFFFFFu, need_band)) {
+        int cnt = 0;
+        for (int cb = 0; cb * 32 < Npad; ++cb) {
+          float v[32];
+          __syncwarp();
+          tmem_ld32(tD + lrow + cb * 32, v);
+          const float4* aj4 = reinterpret_cast<const float4*>(sAj + cb * 32);
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            const float4 A4 = aj4[e >> 2];
+            const float d4[4] = {fmaf(-2.0f, v[e], A4.x), fmaf(-2.0f, v[e + 1], A4.y), fmaf(-2.0f, v[e + 2], A4.z),
+                                 fmaf(-2.0f, v[e + 3], A4.w)};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              if (need_band && d4[i] <= lim) {
+                if (cnt < kBand) myl[1 + cnt] = (uint8_t)(cb * 32 + e + i);
+                ++cnt;
+              }
+          }
+        }
+        if (need_band) n = cnt <= kBand ? cnt : kRecAll;
+      }
+      myl[0] = (uint8_t)n;
+      const int64_t t = (int64_t)tile * 128 + row;
+      if (t < a.N) {
+        uint8_t* dst = head + L.tiles_off + (int64_t)tile * L.tile_bytes + o_rec + row * 32;
+        reinterpret_cast<uint4*>(dst)[0] = reinterpret_cast<const uint4*>(myl)[0];
+        reinterpret_cast<uint4*>(dst)[1] = reinterpret_cast<const uint4*>(myl)[1];
+      }
+      tc_fence_before();
+      named_bar_sync(1 + g, 128);
+      if (flagB[g]) break;
+    }
+    __syncthreads();
+    if (flagA[0] | flagA[1] | flagB[0] | flagB[1]) break;
+    s0 = s1;
+  }
+  if (tid == 0 && (flagA[0] | flagA[1] | flagB[0] | flagB[1]))
+    atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_TIMEOUT);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tbase, 512);
+  }
+}
+
+// ============================================================================
+// Kernel 2: exact quantisation, thread = token
+// ============================================================================
+constexpr int QNT = 128;
+template <int R>
+struct QSmem {
+  static constexpr int K = 0;                                 // token tile, bf16, swizzled
+  static constexpr int U = 32768;                             // U [128][R] fp32
+  static constexpr int G = U + (R > 0 ? 128 * R * 4 : 0);     // U^T W U [R][R] fp32
+  static constexpr int W = G + (R > 0 ? R * R * 4 : 0);       // w [128] fp32
+  static constexpr int MISC = W + 512;                        // W_g[4], |U|_F^2 and max w per warp
+  static constexpr int BAR = MISC + 128;
+  static constexpr int BYTES = BAR + 64 + 1024;
+};
+
+constexpr float kMagic = 12582912.0f;   // 1.5 * 2^23: (y + kMagic) - kMagic = rint(y) for |y| < 2^22
+constexpr float kTwo23 = 8388608.0f;
+
+// Exact Query-aware distance (Eq. 9) in channel order, one fused
+// multiply-add per term on the rounded square.
+__device__ __forceinline__ float exact_dq(const uint8_t* sK, int row, const __nv_bfloat16* mu, const float* sW) {
+  float acc = 0.0f;
+#pragma unroll 2
+  for (int ch = 0; ch < 16; ++ch) {
+    const uint4 kv = lds16(sK + sw_off(128, row, ch));
+    const uint4 mv = ldg16(mu + ch * 8);
+    const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      uint64_t t2 = sub2(bf2_to_f2(kw[p]), bf2_to_f2(mw[p]));
+      t2 = mul2(t2, t2);
+      float lo, hi;
+      f2unpack(t2, lo, hi);
+      acc = __fmaf_rn(sW[ch * 8 + 2 * p], lo, acc);
+      acc = __fmaf_rn(sW[ch * 8 + 2 * p + 1], hi, acc);
     }
   }
+  return acc;
+}
+
+__device__ __forceinline__ float sel4(const float (&a)[4], int g) {
+  return g == 0 ? a[0] : (g == 1 ? a[1] : (g == 2 ? a[2] : a[3]));
 }
 
 template <int R, int GS>
-cudaError_t launch_rg(const AppendArgs& a, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(append_kernel<R, GS>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+__global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
+    append_quant(const AppendArgs a, const __grid_constant__ CUtensorMap tm_k,
+                 const __grid_constant__ CUtensorMap tm_v) {
+  using S = QSmem<R>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const Layout& L = a.L;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tile = blockIdx.x, h = blockIdx.y;
+  const bool is_key = blockIdx.z == 0;
+  const int64_t t = (int64_t)tile * 128 + tid;
+  const bool valid = t < a.N;
+  const int C = L.C;
+  constexpr int ng = 128 / GS;
+  const int Mc = a.M;
+  const bool all_cand = Mc >= C;
+  const __nv_bfloat16* tab = (is_key ? a.kc : a.vc) + (size_t)h * C * 128;
+  const bool use_w = is_key && a.w != nullptr;
+  const bool psac = R > 0 && is_key && a.U != nullptr;
+  uint8_t* head = a.base + head_offset(L, a.slot, h);
+  uint8_t* tb = head + L.tiles_off + (int64_t)tile * L.tile_bytes;
+
+  const uint8_t* sK = sm + S::K;
+  float* sU = reinterpret_cast<float*>(sm + S::U);
+  float* sG = reinterpret_cast<float*>(sm + S::G);
+  float* sW = reinterpret_cast<float*>(sm + S::W);
+  float* sMisc = reinterpret_cast<float*>(sm + S::MISC);
+  const uint32_t bar = smem_u32(sm + S::BAR);
+
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(bar, 32768);
+    const CUtensorMap* tm = is_key ? &tm_k : &tm_v;
+    tma_load_3d(smem_u32(sm + S::K), tm, 0, h, tile * 128, bar);
+    tma_load_3d(smem_u32(sm + S::K + 16384), tm, 64, h, tile * 128, bar);
+  }
+
+  // The chunk's own tables travel with the slot, stored as binary16 (exact
+  // for bf16 values in the binary16 range), the operand type of the
+  // attention kernel's tensor-core path.
+  if (tile == 0) {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
+    __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
+    for (int i = tid; i < C * 64; i += QNT) {
+      const uint32_t pr = src[i];
+      dst[i] = __floats2half2_rn(__uint_as_float(pr << 16), __uint_as_float(pr & 0xFFFF0000u));
+    }
+    if (psac) {
+      __nv_bfloat16* ut = reinterpret_cast<__nv_bfloat16*>(head + L.ut);
+      const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
+      for (int i = tid; i < R * 128; i += QNT) ut[i] = Uh[(size_t)(i % 128) * R + i / 128];  // U_r^T [r][d]
+    }
+  }
+
+  sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
+  if constexpr (R > 0) {
+    if (psac) {
+      const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
+      for (int i = tid; i < 128 * R; i += QNT) sU[i] = __bfloat162float(Uh[i]);  // [d][r]
+    }
+  }
+  __syncthreads();
+  if (tid < ng) {
+    float Wg = 0.0f;
+    for (int c = tid * GS; c < (tid + 1) * GS; ++c) Wg = __fadd_rn(Wg, sW[c]);
+    sMisc[tid] = Wg;
+  }
+  if constexpr (R > 0) {
+    if (psac) {
+      // U^T W U (any order; it enters only with its error bound), |U|_F^2, max w
+      for (int e = tid; e < R * R; e += QNT) {
+        const int j = e / R, k = e % R;
+        float s = 0.0f;
+        for (int c = 0; c < 128; ++c) s = fmaf(sU[c * R + j] * sW[c], sU[c * R + k], s);
+        sG[e] = s;
+      }
+      float u2 = 0.0f;
+#pragma unroll
+      for (int j = 0; j < R; ++j) u2 = fmaf(sU[tid * R + j], sU[tid * R + j], u2);
+      float wm = sW[tid];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        u2 += __shfl_xor_sync(0xFFFFFFFFu, u2, off);
+        wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, off));
+      }
+      if (lane == 0) {
+        sMisc[8 + warp] = u2;
+        sMisc[12 + warp] = wm;
+      }
+    }
+  }
+  __syncthreads();
+  float Wg[4];
+#pragma unroll
+  for (int gi = 0; gi < 4; ++gi) Wg[gi] = gi < ng ? sMisc[gi] : 0.0f;
+
+  // ---- the filter's record for this token
+  uint32_t rec[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) rec[i] = 0;
+  uint32_t* dcodes = reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_codes : L.v_codes) + tid * 32);
+  if (!all_cand && valid) {
+    const uint4 r0 = ldg16(dcodes), r1 = ldg16(dcodes + 4);
+    rec[0] = r0.x; rec[1] = r0.y; rec[2] = r0.z; rec[3] = r0.w;
+    rec[4] = r1.x; rec[5] = r1.y; rec[6] = r1.z; rec[7] = r1.w;
+  }
+  if (!mbar_wait(bar, 0)) {
+    if (lane == 0) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_TIMEOUT);
+    return;
+  }
+  if (!valid) return;
+
+  // ---- 1. candidates
+  int cand[kMaxFilterM];
+#pragma unroll
+  for (int s = 0; s < kMaxFilterM; ++s) cand[s] = 0;
+  if (!all_cand) {
+    auto rb = [&](int i) -> int { return (int)((rec[i >> 2] >> (8 * (i & 3))) & 0xFFu); };
+    const int n = rb(0);
+    bool idsok = true;
+#pragma unroll
+    for (int i = 1; i <= kBand; ++i)
+      if (i <= n && rb(i) >= C) idsok = false;
+    if (n == Mc && idsok) {
+#pragma unroll
+      for (int s = 0; s < kMaxFilterM; ++s) cand[s] = rb(1 + s);
+    } else {
+      // exact rescoring: the band members, or every centroid
+      float ev[kMaxFilterM];
+      int ej[kMaxFilterM];
+#pragma unroll
+      for (int s = 0; s < kMaxFilterM; ++s) { ev[s] = INFINITY; ej[s] = 0x7FFFFFFF; }
+      float ek = INFINITY;
+      const bool band = n >= Mc && n <= kBand && idsok;  // a band holds at least M members
+      const int n_eval = band ? n : C;
+      for (int m = 0; m < n_eval; ++m) {
+        int j = m;
+        if (band) {
+#pragma unroll
+          for (int i = 0; i < kBand; ++i)
+            if (i == m) j = rb(1 + i);
+        }
+        const float dq = exact_dq(sK, tid, tab + (size_t)j * 128, sW);
+        if (dq < ek) {
+          insert_top(ev, ej, Mc, dq, j);
+          ek = sel_at(ev, Mc - 1);
+        }
+      }
+#pragma unroll
+      for (int s = 0; s < kMaxFilterM; ++s) cand[s] = ej[s];
+    }
+  }
+
+  // ---- 2. QSAC score (Eq. 10, 12) of each candidate, lowest (S, j); the
+  // group minima / maxima of the chosen residual feed the INT2 step.
+  float bestS = INFINITY;
+  int bestj = 0x7FFFFFFF;
+  float bmn[4], bmx[4];
+#pragma unroll
+  for (int gi = 0; gi < 4; ++gi) { bmn[gi] = 0.0f; bmx[gi] = 0.0f; }
+  const int ncand = all_cand ? C : Mc;
+  for (int m = 0; m < ncand; ++m) {
+    int j = m;
+    if (!all_cand) {
+#pragma unroll
+      for (int s = 0; s < kMaxFilterM; ++s)
+        if (s == m) j = cand[s];
+    }
+    const __nv_bfloat16* mr = tab + (size_t)j * 128;
+    float mx[4], mn[4];
+#pragma unroll
+    for (int gi = 0; gi < 4; ++gi) { mx[gi] = -INFINITY; mn[gi] = INFINITY; }
+#pragma unroll
+    for (int ch = 0; ch < 16; ++ch) {
+      const uint4 kv = lds16(sK + sw_off(128, tid, ch));
+      const uint4 mv = ldg16(mr + ch * 8);
+      const int gi = (ch * 8) / GS;
+      const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+      float x[8];
+#pragma unroll
+      for (int p = 0; p < 4; ++p) f2unpack(sub2(bf2_to_f2(kw[p]), bf2_to_f2(mw[p])), x[2 * p], x[2 * p + 1]);
+      mx[gi] = fmax3f(mx[gi], x[0], x[1]);
+      mx[gi] = fmax3f(mx[gi], x[2], x[3]);
+      mx[gi] = fmax3f(mx[gi], x[4], x[5]);
+      mx[gi] = fmax3f(mx[gi], x[6], x[7]);
+      mn[gi] = fmin3(mn[gi], x[0], x[1]);
+      mn[gi] = fmin3(mn[gi], x[2], x[3]);
+      mn[gi] = fmin3(mn[gi], x[4], x[5]);
+      mn[gi] = fmin3(mn[gi], x[6], x[7]);
+    }
+    float Sc = 0.0f;
+#pragma unroll
+    for (int gi = 0; gi < ng; ++gi) {
+      const float Rg = __fsub_rn(mx[gi], mn[gi]);
+      Sc = __fadd_rn(Sc, __fmul_rn(Wg[gi], __fmul_rn(Rg, Rg)));
+    }
+    if (Sc < bestS || (Sc == bestS && j < bestj)) {
+      bestS = Sc;
+      bestj = j;
+#pragma unroll
+      for (int gi = 0; gi < 4; ++gi) { bmn[gi] = mn[gi]; bmx[gi] = mx[gi]; }
+    }
+  }
+  const int id = bestj < C ? bestj : C - 1;
+  const __nv_bfloat16* mr = tab + (size_t)id * 128;
+
+  // ---- 3. INT2 parameters (Eq. 1-2): range of the residual with 0 included
+  float sc[4], inv[4], zf[4];
+  __half sh[4];
+  uint32_t zbyte = 0;
+#pragma unroll
+  for (int gi = 0; gi < 4; ++gi) {
+    sc[gi] = 0.0f; inv[gi] = 0.0f; zf[gi] = 0.0f; sh[gi] = __ushort_as_half(0);
+    if (gi < ng) {
+      const float lo = fminf(0.0f, bmn[gi]), hi = fmaxf(0.0f, bmx[gi]);
+      sh[gi] = __float2half_ru(__fdiv_rn(__fsub_rn(hi, lo), 3.0f));
+      sc[gi] = __half2float(sh[gi]);
+      int zq = 0;
+      if (sc[gi] != 0.0f) {
+        inv[gi] = __frcp_rn(sc[gi]);
+        const int z = (int)rintf(__fmul_rn(-lo, inv[gi]));
+        zq = z < 0 ? 0 : (z > 3 ? 3 : z);
+      }
+      zf[gi] = (float)zq;
+      zbyte |= (uint32_t)zq << (2 * gi);
+    }
+  }
+
+  // ---- 4. one channel pass: INT2 codes; Keys with PSAC also E (Eq. 4, 13),
+  // c = U^T E, v = U^T (w o E) and err0 = sum_c w_c E_c^2, in channel order
+  constexpr int RP = R > 0 ? R / 2 : 1;
+  uint64_t cj[RP], vj[RP];
+#pragma unroll
+  for (int i = 0; i < RP; ++i) { cj[i] = 0; vj[i] = 0; }
+  float err0 = 0.0f;
+  uint32_t cw[8];
+  const uint64_t MAG2 = f2pack(kMagic, kMagic);
+#pragma unroll 1
+  for (int wd = 0; wd < 8; ++wd) {
+    const int gi = (wd * 16) / GS;
+    const float s = sel4(sc, gi), iv = sel4(inv, gi), z = sel4(zf, gi);
+    const uint64_t S2 = f2pack(s, s), Z2 = f2pack(z, z);
+    uint32_t word = 0;
+#pragma unroll
+    for (int hc = 0; hc < 2; ++hc) {
+      const int ch = 2 * wd + hc;
+      const uint4 kv = lds16(sK + sw_off(128, tid, ch));
+      const uint4 mv = ldg16(mr + ch * 8);
+      const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const uint64_t k2 = bf2_to_f2(kw[p]), m2 = bf2_to_f2(mw[p]);
+        float x0, x1;
+        f2unpack(sub2(k2, m2), x0, x1);
+        // y = x * (1/s) rounded on its own (the scalar intrinsic is never fused
+        // into the following add), then rint(y) in both lanes
+        const uint64_t y2 = f2pack(__fmul_rn(x0, iv), __fmul_rn(x1, iv));
+        const uint64_t r2 = sub2(add2(y2, MAG2), MAG2);
+        float q0, q1;
+        f2unpack(add2(r2, Z2), q0, q1);
+        q0 = fminf(fmaxf(q0, 0.0f), 3.0f);
+        q1 = fminf(fmaxf(q1, 0.0f), 3.0f);
+        const uint32_t b0 = __float_as_uint(q0 + kTwo23) & 3u, b1 = __float_as_uint(q1 + kTwo23) & 3u;
+        word |= (b0 | (b1 << 16)) << (8 * hc + 2 * p);
+        if constexpr (R > 0) {
+          if (psac) {
+            // E = k - (mu + (q - z) s), then the channel pair's PSAC terms
+            const uint64_t dq2 = sub2(f2pack(q0, q1), Z2);
+            const uint64_t E2 = sub2(k2, add2(m2, mul2(dq2, S2)));
+            const int c0 = ch * 8 + 2 * p;
+            const uint64_t w2 = *reinterpret_cast<const uint64_t*>(sW + c0);
+            const uint64_t wE2 = mul2(w2, E2);
+            float E0, E1, wE0, wE1;
+            f2unpack(E2, E0, E1);
+            f2unpack(wE2, wE0, wE1);
+            const uint64_t e0 = f2pack(E0, E0), e1 = f2pack(E1, E1);
+            const uint64_t we0 = f2pack(wE0, wE0), we1 = f2pack(wE1, wE1);
+            const uint64_t* u0 = reinterpret_cast<const uint64_t*>(sU + c0 * R);
+            const uint64_t* u1 = reinterpret_cast<const uint64_t*>(sU + (c0 + 1) * R);
+#pragma unroll
+            for (int i = 0; i < RP; ++i) {
+              const uint64_t ua = u0[i];
+              cj[i] = fma2(e0, ua, cj[i]);
+              vj[i] = fma2(ua, we0, vj[i]);
+            }
+#pragma unroll
+            for (int i = 0; i < RP; ++i) {
+              const uint64_t ub = u1[i];
+              cj[i] = fma2(e1, ub, cj[i]);
+              vj[i] = fma2(ub, we1, vj[i]);
+            }
+            float t0, t1, w0, w1;
+            f2unpack(mul2(E2, E2), t0, t1);
+            f2unpack(w2, w0, w1);
+            err0 = __fmaf_rn(w0, t0, err0);
+            err0 = __fmaf_rn(w1, t1, err0);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (i == wd) cw[i] = word;
+  }
+  reinterpret_cast<uint4*>(dcodes)[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+  reinterpret_cast<uint4*>(dcodes)[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+  if constexpr (ng == 4) {
+    uint2 sv;
+    sv.x = (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
+    sv.y = (uint32_t)__half_as_ushort(sh[2]) | ((uint32_t)__half_as_ushort(sh[3]) << 16);
+    *reinterpret_cast<uint2*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 8) = sv;
+  } else {
+    *reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 4) =
+        (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
+  }
+  tb[(is_key ? L.k_ids : L.v_ids) + tid] = (uint8_t)id;
+  {
+    uint8_t* dz = tb + (is_key ? L.k_zeros : L.v_zeros) + (int64_t)tid * L.zb;
+    dz[0] = (uint8_t)zbyte;
+    for (int b = 1; b < L.zb; ++b) dz[b] = 0;
+  }
+
+  // ---- 5. PSAC coefficients (Eq. 13, INT8 with a binary16 row scale) and
+  // the keep rule (Eq. 16), Keys only
+  if constexpr (R > 0) {
+    if (is_key) {
+      int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)tid * R);
+      __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma) + tid;
+      uint32_t cwd[R / 4];
+#pragma unroll
+      for (int i = 0; i < R / 4; ++i) cwd[i] = 0;
+      __half sgh_out = __ushort_as_half(0);
+      if (psac) {
+        float c[R], v[R];
+#pragma unroll
+        for (int i = 0; i < RP; ++i) {
+          f2unpack(cj[i], c[2 * i], c[2 * i + 1]);
+          f2unpack(vj[i], v[2 * i], v[2 * i + 1]);
+        }
+        float amax = 0.0f;
+#pragma unroll
+        for (int j = 0; j < R; ++j) amax = fmaxf(amax, fabsf(c[j]));
+        const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
+        const float sg = __half2float(sgh);
+        const float sinv = sg != 0.0f ? __frcp_rn(sg) : 0.0f;
+        float chat[R];
+        uint32_t tq[R / 4];
+#pragma unroll
+        for (int i = 0; i < R / 4; ++i) tq[i] = 0;
+#pragma unroll
+        for (int j = 0; j < R; ++j) {
+          const float qq = sg != 0.0f ? fminf(fmaxf(rintf(__fmul_rn(c[j], sinv)), -127.0f), 127.0f) : 0.0f;
+          tq[j >> 2] |= ((uint32_t)(int)qq & 0xFFu) << (8 * (j & 3));
+          chat[j] = __fmul_rn(qq, sg);
+        }
+        bool keep = false;  // sigma == 0: chat = 0, so errq == err0 and the rule says no
+        if (sg != 0.0f) {
+          // errq - err0 = chat^T G chat - 2 chat.v with G = U^T W U
+          float quad = 0.0f, cv = 0.0f, cn2 = 0.0f, vn2 = 0.0f;
+#pragma unroll
+          for (int j = 0; j < R; ++j) {
+            float gj = 0.0f;
+#pragma unroll
+            for (int k = 0; k < R; ++k) gj = fmaf(sG[j * R + k], chat[k], gj);
+            quad = fmaf(chat[j], gj, quad);
+            cv = fmaf(chat[j], v[j], cv);
+            cn2 = fmaf(chat[j], chat[j], cn2);
+            vn2 = fmaf(v[j], v[j], vn2);
+          }
+          float UF2 = 0.0f, wmax = 0.0f;
+#pragma unroll
+          for (int i = 0; i < QNT / 32; ++i) {
+            UF2 += sMisc[8 + i];
+            wmax = fmaxf(wmax, sMisc[12 + i]);
+          }
+          const float delta = fmaf(-2.0f, cv, quad);
+          const float eq = fabsf(err0 + delta);
+          const float Q = wmax * UF2 * cn2 * 1.0001f;
+          const float bound =
+              ldexpf(eq + err0 + Q + sqrtf(err0 * Q) + sqrtf(eq * Q) + sqrtf(cn2 * vn2), -14) + 1e-35f;
+          if (delta < -bound) {
+            keep = true;
+          } else if (!(delta > bound)) {
+            // too close to call: the sequential evaluation of both sums
+            float errq = 0.0f, e0 = 0.0f;
+#pragma unroll 1
+            for (int wd = 0; wd < 8; ++wd) {
+              const int gi = (wd * 16) / GS;
+              const float s = sel4(sc, gi), z = sel4(zf, gi);
+              uint32_t word = cw[0];
+#pragma unroll
+              for (int i = 1; i < 8; ++i)
+                if (i == wd) word = cw[i];
+#pragma unroll
+              for (int hc = 0; hc < 2; ++hc) {
+                const int ch = 2 * wd + hc;
+                const uint4 kv = lds16(sK + sw_off(128, tid, ch));
+                const uint4 mv = ldg16(mr + ch * 8);
+                const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  const int c = ch * 8 + e;
+                  const float kf = __uint_as_float((e & 1) ? (kw[e >> 1] & 0xFFFF0000u) : (kw[e >> 1] << 16));
+                  const float mf = __uint_as_float((e & 1) ? (mw[e >> 1] & 0xFFFF0000u) : (mw[e >> 1] << 16));
+                  const int j16 = 8 * hc + e;
+                  const float q = (float)((word >> (16 * (j16 & 1) + 2 * (j16 >> 1))) & 3u);
+                  const float E = __fsub_rn(kf, __fadd_rn(mf, __fmul_rn(__fsub_rn(q, z), s)));
+                  float u = 0.0f;
+#pragma unroll
+                  for (int j = 0; j < R; ++j) u = __fmaf_rn(sU[c * R + j], chat[j], u);
+                  const float ep = __fsub_rn(E, u);
+                  errq = __fmaf_rn(sW[c], __fmul_rn(ep, ep), errq);
+                  e0 = __fmaf_rn(sW[c], __fmul_rn(E, E), e0);
+                }
+              }
+            }
+            keep = errq < e0;
+          }
+        }
+        if (keep) {
+#pragma unroll
+          for (int i = 0; i < R / 4; ++i) cwd[i] = tq[i];
+          sgh_out = sgh;
+        }
+      }
+      if constexpr (R == 8) {
+        *reinterpret_cast<uint2*>(coef) = make_uint2(cwd[0], cwd[1]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < R / 16; ++i)
+          reinterpret_cast<uint4*>(coef)[i] = make_uint4(cwd[4 * i], cwd[4 * i + 1], cwd[4 * i + 2], cwd[4 * i + 3]);
+      }
+      *sig = sgh_out;
+    }
+  }
+}
+
+// ============================================================================
+// Host side
+// ============================================================================
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
+// Tensor map over bf16 tokens x[N][H][128]: boxes of 64 channels x 1 head x
+// 128 tokens, 128-byte swizzle (the layout of one K-major operand block);
+// rows past N read as zeros.
+bool token_map(CUtensorMap* m, const void* x, int64_t N, int H) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {128, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[2] = {256, (cuuint64_t)H * 256};
+  cuuint32_t box[3] = {64, 1, 128};
+  cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(x), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int R, int GS>
+cudaError_t launch_quant(const AppendArgs& a, const CUtensorMap& tk, const CUtensorMap& tv, cudaStream_t st) {
+  constexpr int smem = QSmem<R>::BYTES;
+  cudaError_t e = cudaFuncSetAttribute(append_quant<R, GS>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)((a.N + NT - 1) / NT), (unsigned)a.L.H, 2);
-  append_kernel<R, GS><<<grid, NT, SMEM_BYTES, st>>>(a);
+  dim3 grid((unsigned)((a.N + 127) / 128), (unsigned)a.L.H, 2);
+  append_quant<R, GS><<<grid, QNT, smem, st>>>(a, tk, tv);
   return cudaGetLastError();
 }
 template <int R>
-cudaError_t launch_r(const AppendArgs& a, cudaStream_t st) {
-  return a.L.G == 32 ? launch_rg<R, 32>(a, st) : launch_rg<R, 64>(a, st);
+cudaError_t launch_quant_r(const AppendArgs& a, const CUtensorMap& tk, const CUtensorMap& tv, cudaStream_t st) {
+  return a.L.G == 32 ? launch_quant<R, 32>(a, tk, tv, st) : launch_quant<R, 64>(a, tk, tv, st);
 }
 
 }  // namespace
 
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
   if (a.M > kMaxFilterM && a.M < a.L.C) return launch_append_generic(a, st);
+  alignas(64) CUtensorMap tk, tv;
+  if (!token_map(&tk, a.k, a.N, a.L.H) || !token_map(&tv, a.v, a.N, a.L.H)) return cudaErrorInvalidValue;
+  if (a.M < a.L.C) {
+    int dev = 0, nsm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(append_filter, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
+    if (e != cudaSuccess) return e;
+    const int tiles = (int)((a.N + 127) / 128);
+    const int units = 2 * a.L.H * tiles;
+    const int grid = units < nsm ? units : nsm;
+    append_filter<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   switch (a.L.r) {
-    case 0: return launch_r<0>(a, st);
-    case 8: return launch_r<8>(a, st);
-    case 16: return launch_r<16>(a, st);
-    case 32: return launch_r<32>(a, st);
+    case 0: return launch_quant_r<0>(a, tk, tv, st);
+    case 8: return launch_quant_r<8>(a, tk, tv, st);
+    case 16: return launch_quant_r<16>(a, tk, tv, st);
+    case 32: return launch_quant_r<32>(a, tk, tv, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -9,8 +9,9 @@
 // (blockIdx.z = 1).  Every quantity that decides an integer (distances, QSAC
 // scores, scales, codes, PSAC codes, keep test) is evaluated in fp32 with
 // explicitly rounded operations (__fadd_rn / __fmul_rn / __fdiv_rn, never
-// contracted), summed in channel order, so the packed output is bit-exact
-// against a sequential fp32 evaluation of the same formulas.
+// contracted, and one __fmaf_rn per term of the sums of products), summed in
+// channel order, so the packed output is bit-exact against a sequential fp32
+// evaluation of the same formulas.
 #include "qwm_internal.cuh"
 
 namespace qwm {
@@ -133,9 +134,9 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
 #pragma unroll
       for (int i = 0; i < TT; ++i) {
         float t = __fsub_rn(s.x[i * 128 + 2 * cw], m0);
-        acc[i] = __fadd_rn(acc[i], __fmul_rn(w0, __fmul_rn(t, t)));
+        acc[i] = __fmaf_rn(w0, __fmul_rn(t, t), acc[i]);
         t = __fsub_rn(s.x[i * 128 + 2 * cw + 1], m1);
-        acc[i] = __fadd_rn(acc[i], __fmul_rn(w1, __fmul_rn(t, t)));
+        acc[i] = __fmaf_rn(w1, __fmul_rn(t, t), acc[i]);
       }
     }
 #pragma unroll
@@ -287,7 +288,7 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
         __syncwarp();
         float cj = 0.0f;
         if (lane < r)
-          for (int c = 0; c < 128; ++c) cj = __fadd_rn(cj, __fmul_rn(se[c], bf2f(s.U[c * r + lane])));
+          for (int c = 0; c < 128; ++c) cj = __fmaf_rn(se[c], bf2f(s.U[c * r + lane]), cj);
         float amax = lane < r ? fabsf(cj) : 0.0f;
 #pragma unroll
         for (int off = 16; off; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, off));
@@ -310,19 +311,19 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
           float u = 0.0f;
           for (int j = 0; j < r; ++j) {
             const float chj = __shfl_sync(0xFFFFFFFFu, ch, j);
-            u = __fadd_rn(u, __fmul_rn(bf2f(s.U[c * r + j]), chj));
+            u = __fmaf_rn(bf2f(s.U[c * r + j]), chj, u);
           }
           const float ep = __fsub_rn(E[e], u);
-          stq[c] = __fmul_rn(s.w[c], __fmul_rn(ep, ep));
-          st0[c] = __fmul_rn(s.w[c], __fmul_rn(E[e], E[e]));
+          stq[c] = __fmul_rn(ep, ep);
+          st0[c] = __fmul_rn(E[e], E[e]);
         }
         __syncwarp();
         int keep = 0;
         if (lane == 0) {
           float errq = 0.0f, err0 = 0.0f;
           for (int c = 0; c < 128; ++c) {
-            errq = __fadd_rn(errq, stq[c]);
-            err0 = __fadd_rn(err0, st0[c]);
+            errq = __fmaf_rn(s.w[c], stq[c], errq);
+            err0 = __fmaf_rn(s.w[c], st0[c], err0);
           }
           keep = errq < err0;
         }
