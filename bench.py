@@ -79,10 +79,17 @@ class ClockSampler:
             os.close(fd)
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=self.fh, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
+            return
+        # the sampler is live once its first row is out; then the timed region starts
+        t_end = time.time() + 5.0
+        while time.time() < t_end and self.proc.poll() is None:
+            if os.path.getsize(self.path) > 0:
+                break
+            time.sleep(0.02)
 
     def stop(self):
         if self.proc is None:
@@ -265,7 +272,9 @@ def run_gpu(args, wl, rank, world):
                      "frac": round(att_tflops / pk["bf16_tflops_sustained"], 4), "traffic": None,
                      "peak_src": pk["src"] + " sustained bf16"},
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 2 * args.steps,
+        # attend: one kernel; append: the candidate filter and the quantize kernel
+        # when M <= 8 and M < C, a single kernel otherwise
+        "gpu_launches": (1 + (2 if (M < C and M <= 8) else 1)) * args.steps,
         "clocks": clk,
     }
     return res
@@ -356,7 +365,7 @@ def run_reference(args, wl):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="qwm", choices=["qwm", "reference"])
     ap.add_argument("--workload", default="wan14b_layer")

@@ -161,7 +161,9 @@ QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, const void* 
 /* Quantize one finished chunk and append it to the cache (Sec. 4.1 QSAC,
  * Sec. 2 Eq. 1-4 INT2 residuals, Sec. 4.2 Eq. 13/16 PSAC, App. D.1 packing).
  * k, v: bf16 [N][H][d], 1 <= N <= tokens_per_chunk.  k_centroids,
- * v_centroids: bf16 [H][C][d] (this chunk's tables; copied into the slot).
+ * v_centroids: bf16 [H][C][d], 32-byte aligned (this chunk's tables; copied
+ * into the slot); a table that is only 16-byte aligned returns
+ * QWM_ERR_INVALID_ARG.
  * w: fp32 [H][d] channel sensitivity weights (Eq. 8) or NULL for w = 1 (the
  * cold-start rule of App. C.3).  U: bf16 [H][d][r] principal Query basis
  * (Eq. 15) or NULL to store no PSAC correction (cold start).  Keys: top-M

@@ -56,6 +56,12 @@ constexpr int kRecAll = 255;      // record: rescore every centroid
 
 __device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
 __device__ __forceinline__ uint4 lds16(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
+// 32-byte read-only global load (address 32-byte aligned): one whole sector.
+__device__ __forceinline__ void ldg32(const void* p, uint32_t (&r)[8]) {
+  asm volatile("ld.global.nc.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+               : "l"(p));
+}
 
 // Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in a
 // pair of 128-byte-swizzled blocks of `rows` rows x 64 two-byte elements.
@@ -271,16 +277,19 @@ __global__ void __launch_bounds__(FNT, 1)
       ph_mma ^= 1;
       tc_fence_after();
 
-      // ---- M+1 smallest dt_j of this row
+      // ---- selection over dt_j = A_j - 2 D_j (the TMEM reads are
+      // warp-collective, every other step is per row).
+      //   1. the minima of 16 interleaved column groups (column j in group
+      //      j % 16); their (M+1)-th smallest, T, bounds the (M+1)-th
+      //      smallest dt from above;
+      //   2. the few columns with dt <= T go, in ascending j, to a per-row
+      //      list in this group's A tile (free once the MMA has completed);
+      //   3. the M+1 smallest of the list are the M+1 smallest of the row.
       constexpr int CAP = kMaxFilterM + 1;
-      float tv[CAP];
-      int tj[CAP];
-#pragma unroll
-      for (int s = 0; s < CAP; ++s) { tv[s] = INFINITY; tj[s] = 0x7FFFFFFF; }
-      float thr = INFINITY;  // the (M+1)-th smallest so far
-      for (int cb = 0; cb * 32 < Npad; ++cb) {
-        float v[32];
-        __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the insertions
+      constexpr int kList = 32;
+      const int nchunk = (Npad + 31) >> 5;
+      auto load_dt = [&](int cb, float (&v)[32]) {
+        __syncwarp();
         tmem_ld32(tD + lrow + cb * 32, v);
         const float4* aj4 = reinterpret_cast<const float4*>(sAj + cb * 32);
 #pragma unroll
@@ -291,26 +300,67 @@ __global__ void __launch_bounds__(FNT, 1)
           v[e + 2] = fmaf(-2.0f, v[e + 2], A4.z);
           v[e + 3] = fmaf(-2.0f, v[e + 3], A4.w);
         }
-        float mn = fmin3(v[0], v[1], v[2]);
+      };
+      float gm[16];
 #pragma unroll
-        for (int e = 3; e < 31; e += 2) mn = fmin3(mn, v[e], v[e + 1]);
-        mn = fminf(mn, v[31]);
-        if (mn < thr) {
+      for (int i = 0; i < 16; ++i) gm[i] = INFINITY;
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            if (v[e] < thr) {
-              insert_top(tv, tj, Mc + 1, v[e], cb * 32 + e);
-              thr = sel_at(tv, Mc);
-            }
-          }
+      for (int cb = 0; cb < 8; ++cb) {
+        if (cb < nchunk) {
+          float v[32];
+          load_dt(cb, v);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) gm[e] = fmin3(gm[e], v[e], v[e + 16]);
         }
       }
-      const float kth = sel_at(tv, Mc - 1);
+      float tq[CAP];
+#pragma unroll
+      for (int i = 0; i < CAP; ++i) tq[i] = INFINITY;
+#pragma unroll
+      for (int gi = 0; gi < 16; ++gi) {  // sorted insertion, every slot from the old values
+        const float x = gm[gi];
+#pragma unroll
+        for (int i = CAP - 1; i > 0; --i) tq[i] = fmaxf(tq[i - 1], fminf(tq[i], x));
+        tq[0] = fminf(tq[0], x);
+      }
+      const float T = sel_at(tq, Mc);
+
+      // [kList] entries of (dt, column) per row, slot-swizzled against bank conflicts
+      uint2* lst = reinterpret_cast<uint2*>(sA + row * 256);
+      const int sw = row & 31;
+      int cnt = 0;
+#pragma unroll 1
+      for (int cb = 0; cb < nchunk; ++cb) {
+        float v[32];
+        load_dt(cb, v);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          // branch-free: every column is written at the current slot, which
+          // advances only when the column is taken
+          lst[(cnt < kList ? cnt : kList - 1) ^ sw] = make_uint2(__float_as_uint(v[e]), (uint32_t)(cb * 32 + e));
+          cnt += v[e] <= T ? 1 : 0;
+        }
+      }
+      float tv[CAP];
+      int tj[CAP];
+#pragma unroll
+      for (int i = 0; i < CAP; ++i) { tv[i] = INFINITY; tj[i] = 0x7FFFFFFF; }
+      const int mc = cnt < kList ? cnt : kList;
+      const int wmx = __reduce_max_sync(0xFFFFFFFFu, mc);
+      for (int i = 0; i < wmx; ++i)
+        if (i < mc) {
+          const uint2 en = lst[i ^ sw];
+          insert_top(tv, tj, Mc + 1, __uint_as_float(en.x), (int)en.y);
+        }
+
+      const float kth = sel_at(tv, Mc - 1), nxt = sel_at(tv, Mc);
       const float kn = sqrtf(kn2);
       const float Bb = ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
       const float lim = kth + 2.0f * Bb;
-      const bool over = !(kmx <= 65504.0f) || !(kn2 < INFINITY) || !(lim < INFINITY);
-      const bool decided = !over && thr > lim;
+      // a list overflow (more than kList columns at or below T) or a row out
+      // of the binary16 range is left to the exact rescoring of every centroid
+      const bool over = cnt > kList || !(kmx <= 65504.0f) || !(kn2 < INFINITY) || !(lim < INFINITY);
+      const bool decided = !over && nxt > lim;
       int n = over ? kRecAll : Mc;
       if (decided) {
 #pragma unroll
@@ -318,30 +368,35 @@ __global__ void __launch_bounds__(FNT, 1)
           if (s < Mc) myl[1 + s] = (uint8_t)tj[s];
       }
       // The band (every j with dt_j <= kth + 2B, ascending j) of the rows
-      // that are not decided; the TMEM reads are warp-collective, so the
-      // whole warp walks the row blocks whenever one of its rows needs it.
+      // that are not decided: from the list when it covers the band
+      // (lim <= T), otherwise from all columns.
       const bool need_band = !over && !decided;
-      if (__any_sync(0xFFFFFFFFu, need_band)) {
-        int cnt = 0;
-        for (int cb = 0; cb * 32 < Npad; ++cb) {
+      if (need_band && lim <= T) {
+        int c2 = 0;
+        for (int i = 0; i < mc; ++i) {
+          const uint2 en = lst[i ^ sw];
+          const bool take = __uint_as_float(en.x) <= lim;
+          const int sl = c2 < kBand ? c2 : kBand - 1;
+          if (take) myl[1 + sl] = (uint8_t)en.y;
+          c2 += take ? 1 : 0;
+        }
+        n = c2 <= kBand ? c2 : kRecAll;
+      }
+      const bool need_scan = need_band && !(lim <= T);
+      if (__any_sync(0xFFFFFFFFu, need_scan)) {
+        int c2 = 0;
+        for (int cb = 0; cb < nchunk; ++cb) {
           float v[32];
-          __syncwarp();
-          tmem_ld32(tD + lrow + cb * 32, v);
-          const float4* aj4 = reinterpret_cast<const float4*>(sAj + cb * 32);
+          load_dt(cb, v);
 #pragma unroll
-          for (int e = 0; e < 32; e += 4) {
-            const float4 A4 = aj4[e >> 2];
-            const float d4[4] = {fmaf(-2.0f, v[e], A4.x), fmaf(-2.0f, v[e + 1], A4.y), fmaf(-2.0f, v[e + 2], A4.z),
-                                 fmaf(-2.0f, v[e + 3], A4.w)};
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              if (need_band && d4[i] <= lim) {
-                if (cnt < kBand) myl[1 + cnt] = (uint8_t)(cb * 32 + e + i);
-                ++cnt;
-              }
+          for (int e = 0; e < 32; ++e) {
+            const bool take = need_scan && v[e] <= lim;
+            const int sl = c2 < kBand ? c2 : kBand - 1;
+            if (take) myl[1 + sl] = (uint8_t)(cb * 32 + e);
+            c2 += take ? 1 : 0;
           }
         }
-        if (need_band) n = cnt <= kBand ? cnt : kRecAll;
+        if (need_scan) n = c2 <= kBand ? c2 : kRecAll;
       }
       myl[0] = (uint8_t)n;
       const int64_t t = (int64_t)tile * 128 + row;
@@ -350,6 +405,7 @@ __global__ void __launch_bounds__(FNT, 1)
         reinterpret_cast<uint4*>(dst)[0] = reinterpret_cast<const uint4*>(myl)[0];
         reinterpret_cast<uint4*>(dst)[1] = reinterpret_cast<const uint4*>(myl)[1];
       }
+      fence_proxy_async_smem();  // the list lived in the A tile, which the next copy overwrites
       tc_fence_before();
       named_bar_sync(1 + g, 128);
       if (flagB[g]) break;
@@ -378,11 +434,14 @@ struct QSmem {
   static constexpr int U = 32768;                             // U [128][R] fp32
   static constexpr int G = U + (R > 0 ? 128 * R * 4 : 0);     // U^T W U [R][R] fp32
   static constexpr int W = G + (R > 0 ? R * R * 4 : 0);       // w [128] fp32
-  static constexpr int MISC = W + 512;                        // W_g[4], |U|_F^2 and max w per warp
-  static constexpr int BAR = MISC + 128;
+  static constexpr int MISC = W + 512;                        // W_g[4], |U|_F^2 and max w per warp, list count
+  static constexpr int RS = MISC + 128;                       // rescoring list: [kRsCap] (row, j) u16
+  static constexpr int RSD = RS + 2 * 512;                    //   and their distances, fp32
+  static constexpr int BAR = RSD + 4 * 512;
   static constexpr int BYTES = BAR + 64 + 1024;
 };
 
+constexpr int kRsCap = 512;             // (token, centroid) pairs rescored together per tile
 constexpr float kMagic = 12582912.0f;   // 1.5 * 2^23: (y + kMagic) - kMagic = rint(y) for |y| < 2^22
 constexpr float kTwo23 = 8388608.0f;
 
@@ -390,19 +449,20 @@ constexpr float kTwo23 = 8388608.0f;
 // multiply-add per term on the rounded square.
 __device__ __forceinline__ float exact_dq(const uint8_t* sK, int row, const __nv_bfloat16* mu, const float* sW) {
   float acc = 0.0f;
-#pragma unroll 2
-  for (int ch = 0; ch < 16; ++ch) {
-    const uint4 kv = lds16(sK + sw_off(128, row, ch));
-    const uint4 mv = ldg16(mu + ch * 8);
-    const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll 4
+  for (int cc = 0; cc < 8; ++cc) {
+    uint32_t mw[8];
+    ldg32(mu + cc * 16, mw);
+    const uint4 ka = lds16(sK + sw_off(128, row, 2 * cc)), kb = lds16(sK + sw_off(128, row, 2 * cc + 1));
+    const uint32_t kw[8] = {ka.x, ka.y, ka.z, ka.w, kb.x, kb.y, kb.z, kb.w};
 #pragma unroll
-    for (int p = 0; p < 4; ++p) {
+    for (int p = 0; p < 8; ++p) {
       uint64_t t2 = sub2(bf2_to_f2(kw[p]), bf2_to_f2(mw[p]));
       t2 = mul2(t2, t2);
       float lo, hi;
       f2unpack(t2, lo, hi);
-      acc = __fmaf_rn(sW[ch * 8 + 2 * p], lo, acc);
-      acc = __fmaf_rn(sW[ch * 8 + 2 * p + 1], hi, acc);
+      acc = __fmaf_rn(sW[cc * 16 + 2 * p], lo, acc);
+      acc = __fmaf_rn(sW[cc * 16 + 2 * p + 1], hi, acc);
     }
   }
   return acc;
@@ -415,438 +475,567 @@ __device__ __forceinline__ float sel4(const float (&a)[4], int g) {
 template <int R, int GS>
 __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
     append_quant(const AppendArgs a, const __grid_constant__ CUtensorMap tm_k,
-                 const __grid_constant__ CUtensorMap tm_v) {
+                 const __grid_constant__ CUtensorMap tm_v, int tiles, int units, int nsm, int cps) {
   using S = QSmem<R>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const Layout& L = a.L;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int tile = blockIdx.x, h = blockIdx.y;
-  const bool is_key = blockIdx.z == 0;
-  const int64_t t = (int64_t)tile * 128 + tid;
-  const bool valid = t < a.N;
-  const int C = L.C;
+  const int H = L.H, C = L.C;
   constexpr int ng = 128 / GS;
+  constexpr int RP = R > 0 ? R / 2 : 1;
   const int Mc = a.M;
   const bool all_cand = Mc >= C;
-  const __nv_bfloat16* tab = (is_key ? a.kc : a.vc) + (size_t)h * C * 128;
-  const bool use_w = is_key && a.w != nullptr;
-  const bool psac = R > 0 && is_key && a.U != nullptr;
-  uint8_t* head = a.base + head_offset(L, a.slot, h);
-  uint8_t* tb = head + L.tiles_off + (int64_t)tile * L.tile_bytes;
 
   const uint8_t* sK = sm + S::K;
   float* sU = reinterpret_cast<float*>(sm + S::U);
   float* sG = reinterpret_cast<float*>(sm + S::G);
   float* sW = reinterpret_cast<float*>(sm + S::W);
   float* sMisc = reinterpret_cast<float*>(sm + S::MISC);
+  int* sRsCount = reinterpret_cast<int*>(sm + S::MISC + 64);
+  uint16_t* sRsPair = reinterpret_cast<uint16_t*>(sm + S::RS);
+  float* sRsDq = reinterpret_cast<float*>(sm + S::RSD);
   const uint32_t bar = smem_u32(sm + S::BAR);
 
+  // Work unit u = (side * H + h) * tiles + tile; this CTA takes the
+  // contiguous run [u0, u1), so its per-(head, side) setup is redone only
+  // where the run crosses into the next head or side, and the head's
+  // centroid table stays hot in L1.
+  // With one full wave (nsm * cps CTAs), CTA b is taken to run on SM
+  // b % nsm, and the cps CTAs of one SM get adjacent runs (one head's table).
+  int li = blockIdx.x;
+  if ((int)gridDim.x == nsm * cps) li = (li % nsm) * cps + li / nsm;
+  const int u0 = (int)((int64_t)li * units / gridDim.x);
+  const int u1 = (int)((int64_t)(li + 1) * units / gridDim.x);
+  auto issue_tile = [&](int u) {
+    const int pr = u / tiles, tl = u - pr * tiles;
+    const CUtensorMap* tm = pr < H ? &tm_k : &tm_v;
+    mbar_arrive_expect_tx(bar, 32768);
+    tma_load_3d(smem_u32(sm + S::K), tm, 0, pr % H, tl * 128, bar);
+    tma_load_3d(smem_u32(sm + S::K + 16384), tm, 64, pr % H, tl * 128, bar);
+  };
   if (tid == 0) {
     mbar_init(bar, 1);
     fence_mbar_init();
-    mbar_arrive_expect_tx(bar, 32768);
-    const CUtensorMap* tm = is_key ? &tm_k : &tm_v;
-    tma_load_3d(smem_u32(sm + S::K), tm, 0, h, tile * 128, bar);
-    tma_load_3d(smem_u32(sm + S::K + 16384), tm, 64, h, tile * 128, bar);
+    if (u0 < u1) issue_tile(u0);
   }
+  uint32_t ph = 0;
+  int cur_pair = -1;
 
-  // The chunk's own tables travel with the slot, stored as binary16 (exact
-  // for bf16 values in the binary16 range), the operand type of the
-  // attention kernel's tensor-core path.
-  if (tile == 0) {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
-    __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
-    for (int i = tid; i < C * 64; i += QNT) {
-      const uint32_t pr = src[i];
-      dst[i] = __floats2half2_rn(__uint_as_float(pr << 16), __uint_as_float(pr & 0xFFFF0000u));
-    }
-    if (psac) {
-      __nv_bfloat16* ut = reinterpret_cast<__nv_bfloat16*>(head + L.ut);
-      const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
-      for (int i = tid; i < R * 128; i += QNT) ut[i] = Uh[(size_t)(i % 128) * R + i / 128];  // U_r^T [r][d]
-    }
-  }
+  for (int u = u0; u < u1; ++u) {
+    const int pair = u / tiles;
+    const int tile = u - pair * tiles, h = pair % H;
+    const bool is_key = pair < H;
+    const int64_t t = (int64_t)tile * 128 + tid;
+    const bool valid = t < a.N;
+    const __nv_bfloat16* tab = (is_key ? a.kc : a.vc) + (size_t)h * C * 128;
+    const bool use_w = is_key && a.w != nullptr;
+    const bool psac = R > 0 && is_key && a.U != nullptr;
+    uint8_t* head = a.base + head_offset(L, a.slot, h);
+    uint8_t* tb = head + L.tiles_off + (int64_t)tile * L.tile_bytes;
+    const __nv_bfloat16* xr = (is_key ? a.k : a.v) + ((size_t)(valid ? t : 0) * H + h) * 128;
 
-  sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
-  if constexpr (R > 0) {
-    if (psac) {
-      const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
-      for (int i = tid; i < 128 * R; i += QNT) sU[i] = __bfloat162float(Uh[i]);  // [d][r]
-    }
-  }
-  __syncthreads();
-  if (tid < ng) {
-    float Wg = 0.0f;
-    for (int c = tid * GS; c < (tid + 1) * GS; ++c) Wg = __fadd_rn(Wg, sW[c]);
-    sMisc[tid] = Wg;
-  }
-  if constexpr (R > 0) {
-    if (psac) {
-      // U^T W U (any order; it enters only with its error bound), |U|_F^2, max w
-      for (int e = tid; e < R * R; e += QNT) {
-        const int j = e / R, k = e % R;
-        float s = 0.0f;
-        for (int c = 0; c < 128; ++c) s = fmaf(sU[c * R + j] * sW[c], sU[c * R + k], s);
-        sG[e] = s;
+    // The chunk's own tables travel with the slot, stored as binary16 (exact
+    // for bf16 values in the binary16 range), the operand type of the
+    // attention kernel's tensor-core path.
+    if (tile == 0) {
+      const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
+      __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
+      for (int i = tid; i < C * 64; i += QNT) {
+        const uint32_t pr = src[i];
+        dst[i] = __floats2half2_rn(__uint_as_float(pr << 16), __uint_as_float(pr & 0xFFFF0000u));
       }
-      float u2 = 0.0f;
-#pragma unroll
-      for (int j = 0; j < R; ++j) u2 = fmaf(sU[tid * R + j], sU[tid * R + j], u2);
-      float wm = sW[tid];
-#pragma unroll
-      for (int off = 16; off; off >>= 1) {
-        u2 += __shfl_xor_sync(0xFFFFFFFFu, u2, off);
-        wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, off));
-      }
-      if (lane == 0) {
-        sMisc[8 + warp] = u2;
-        sMisc[12 + warp] = wm;
-      }
-    }
-  }
-  __syncthreads();
-  float Wg[4];
-#pragma unroll
-  for (int gi = 0; gi < 4; ++gi) Wg[gi] = gi < ng ? sMisc[gi] : 0.0f;
-
-  // ---- the filter's record for this token
-  uint32_t rec[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) rec[i] = 0;
-  uint32_t* dcodes = reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_codes : L.v_codes) + tid * 32);
-  if (!all_cand && valid) {
-    const uint4 r0 = ldg16(dcodes), r1 = ldg16(dcodes + 4);
-    rec[0] = r0.x; rec[1] = r0.y; rec[2] = r0.z; rec[3] = r0.w;
-    rec[4] = r1.x; rec[5] = r1.y; rec[6] = r1.z; rec[7] = r1.w;
-  }
-  if (!mbar_wait(bar, 0)) {
-    if (lane == 0) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_TIMEOUT);
-    return;
-  }
-  if (!valid) return;
-
-  // ---- 1. candidates
-  int cand[kMaxFilterM];
-#pragma unroll
-  for (int s = 0; s < kMaxFilterM; ++s) cand[s] = 0;
-  if (!all_cand) {
-    auto rb = [&](int i) -> int { return (int)((rec[i >> 2] >> (8 * (i & 3))) & 0xFFu); };
-    const int n = rb(0);
-    bool idsok = true;
-#pragma unroll
-    for (int i = 1; i <= kBand; ++i)
-      if (i <= n && rb(i) >= C) idsok = false;
-    if (n == Mc && idsok) {
-#pragma unroll
-      for (int s = 0; s < kMaxFilterM; ++s) cand[s] = rb(1 + s);
-    } else {
-      // exact rescoring: the band members, or every centroid
-      float ev[kMaxFilterM];
-      int ej[kMaxFilterM];
-#pragma unroll
-      for (int s = 0; s < kMaxFilterM; ++s) { ev[s] = INFINITY; ej[s] = 0x7FFFFFFF; }
-      float ek = INFINITY;
-      const bool band = n >= Mc && n <= kBand && idsok;  // a band holds at least M members
-      const int n_eval = band ? n : C;
-      for (int m = 0; m < n_eval; ++m) {
-        int j = m;
-        if (band) {
-#pragma unroll
-          for (int i = 0; i < kBand; ++i)
-            if (i == m) j = rb(1 + i);
-        }
-        const float dq = exact_dq(sK, tid, tab + (size_t)j * 128, sW);
-        if (dq < ek) {
-          insert_top(ev, ej, Mc, dq, j);
-          ek = sel_at(ev, Mc - 1);
-        }
-      }
-#pragma unroll
-      for (int s = 0; s < kMaxFilterM; ++s) cand[s] = ej[s];
-    }
-  }
-
-  // ---- 2. QSAC score (Eq. 10, 12) of each candidate, lowest (S, j); the
-  // group minima / maxima of the chosen residual feed the INT2 step.
-  float bestS = INFINITY;
-  int bestj = 0x7FFFFFFF;
-  float bmn[4], bmx[4];
-#pragma unroll
-  for (int gi = 0; gi < 4; ++gi) { bmn[gi] = 0.0f; bmx[gi] = 0.0f; }
-  const int ncand = all_cand ? C : Mc;
-  for (int m = 0; m < ncand; ++m) {
-    int j = m;
-    if (!all_cand) {
-#pragma unroll
-      for (int s = 0; s < kMaxFilterM; ++s)
-        if (s == m) j = cand[s];
-    }
-    const __nv_bfloat16* mr = tab + (size_t)j * 128;
-    float mx[4], mn[4];
-#pragma unroll
-    for (int gi = 0; gi < 4; ++gi) { mx[gi] = -INFINITY; mn[gi] = INFINITY; }
-#pragma unroll
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 kv = lds16(sK + sw_off(128, tid, ch));
-      const uint4 mv = ldg16(mr + ch * 8);
-      const int gi = (ch * 8) / GS;
-      const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
-      float x[8];
-#pragma unroll
-      for (int p = 0; p < 4; ++p) f2unpack(sub2(bf2_to_f2(kw[p]), bf2_to_f2(mw[p])), x[2 * p], x[2 * p + 1]);
-      mx[gi] = fmax3f(mx[gi], x[0], x[1]);
-      mx[gi] = fmax3f(mx[gi], x[2], x[3]);
-      mx[gi] = fmax3f(mx[gi], x[4], x[5]);
-      mx[gi] = fmax3f(mx[gi], x[6], x[7]);
-      mn[gi] = fmin3(mn[gi], x[0], x[1]);
-      mn[gi] = fmin3(mn[gi], x[2], x[3]);
-      mn[gi] = fmin3(mn[gi], x[4], x[5]);
-      mn[gi] = fmin3(mn[gi], x[6], x[7]);
-    }
-    float Sc = 0.0f;
-#pragma unroll
-    for (int gi = 0; gi < ng; ++gi) {
-      const float Rg = __fsub_rn(mx[gi], mn[gi]);
-      Sc = __fadd_rn(Sc, __fmul_rn(Wg[gi], __fmul_rn(Rg, Rg)));
-    }
-    if (Sc < bestS || (Sc == bestS && j < bestj)) {
-      bestS = Sc;
-      bestj = j;
-#pragma unroll
-      for (int gi = 0; gi < 4; ++gi) { bmn[gi] = mn[gi]; bmx[gi] = mx[gi]; }
-    }
-  }
-  const int id = bestj < C ? bestj : C - 1;
-  const __nv_bfloat16* mr = tab + (size_t)id * 128;
-
-  // ---- 3. INT2 parameters (Eq. 1-2): range of the residual with 0 included
-  float sc[4], inv[4], zf[4];
-  __half sh[4];
-  uint32_t zbyte = 0;
-#pragma unroll
-  for (int gi = 0; gi < 4; ++gi) {
-    sc[gi] = 0.0f; inv[gi] = 0.0f; zf[gi] = 0.0f; sh[gi] = __ushort_as_half(0);
-    if (gi < ng) {
-      const float lo = fminf(0.0f, bmn[gi]), hi = fmaxf(0.0f, bmx[gi]);
-      sh[gi] = __float2half_ru(__fdiv_rn(__fsub_rn(hi, lo), 3.0f));
-      sc[gi] = __half2float(sh[gi]);
-      int zq = 0;
-      if (sc[gi] != 0.0f) {
-        inv[gi] = __frcp_rn(sc[gi]);
-        const int z = (int)rintf(__fmul_rn(-lo, inv[gi]));
-        zq = z < 0 ? 0 : (z > 3 ? 3 : z);
-      }
-      zf[gi] = (float)zq;
-      zbyte |= (uint32_t)zq << (2 * gi);
-    }
-  }
-
-  // ---- 4. one channel pass: INT2 codes; Keys with PSAC also E (Eq. 4, 13),
-  // c = U^T E, v = U^T (w o E) and err0 = sum_c w_c E_c^2, in channel order
-  constexpr int RP = R > 0 ? R / 2 : 1;
-  uint64_t cj[RP], vj[RP];
-#pragma unroll
-  for (int i = 0; i < RP; ++i) { cj[i] = 0; vj[i] = 0; }
-  float err0 = 0.0f;
-  uint32_t cw[8];
-  const uint64_t MAG2 = f2pack(kMagic, kMagic);
-#pragma unroll 1
-  for (int wd = 0; wd < 8; ++wd) {
-    const int gi = (wd * 16) / GS;
-    const float s = sel4(sc, gi), iv = sel4(inv, gi), z = sel4(zf, gi);
-    const uint64_t S2 = f2pack(s, s), Z2 = f2pack(z, z);
-    uint32_t word = 0;
-#pragma unroll
-    for (int hc = 0; hc < 2; ++hc) {
-      const int ch = 2 * wd + hc;
-      const uint4 kv = lds16(sK + sw_off(128, tid, ch));
-      const uint4 mv = ldg16(mr + ch * 8);
-      const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
-#pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const uint64_t k2 = bf2_to_f2(kw[p]), m2 = bf2_to_f2(mw[p]);
-        float x0, x1;
-        f2unpack(sub2(k2, m2), x0, x1);
-        // y = x * (1/s) rounded on its own (the scalar intrinsic is never fused
-        // into the following add), then rint(y) in both lanes
-        const uint64_t y2 = f2pack(__fmul_rn(x0, iv), __fmul_rn(x1, iv));
-        const uint64_t r2 = sub2(add2(y2, MAG2), MAG2);
-        float q0, q1;
-        f2unpack(add2(r2, Z2), q0, q1);
-        q0 = fminf(fmaxf(q0, 0.0f), 3.0f);
-        q1 = fminf(fmaxf(q1, 0.0f), 3.0f);
-        const uint32_t b0 = __float_as_uint(q0 + kTwo23) & 3u, b1 = __float_as_uint(q1 + kTwo23) & 3u;
-        word |= (b0 | (b1 << 16)) << (8 * hc + 2 * p);
-        if constexpr (R > 0) {
-          if (psac) {
-            // E = k - (mu + (q - z) s), then the channel pair's PSAC terms
-            const uint64_t dq2 = sub2(f2pack(q0, q1), Z2);
-            const uint64_t E2 = sub2(k2, add2(m2, mul2(dq2, S2)));
-            const int c0 = ch * 8 + 2 * p;
-            const uint64_t w2 = *reinterpret_cast<const uint64_t*>(sW + c0);
-            const uint64_t wE2 = mul2(w2, E2);
-            float E0, E1, wE0, wE1;
-            f2unpack(E2, E0, E1);
-            f2unpack(wE2, wE0, wE1);
-            const uint64_t e0 = f2pack(E0, E0), e1 = f2pack(E1, E1);
-            const uint64_t we0 = f2pack(wE0, wE0), we1 = f2pack(wE1, wE1);
-            const uint64_t* u0 = reinterpret_cast<const uint64_t*>(sU + c0 * R);
-            const uint64_t* u1 = reinterpret_cast<const uint64_t*>(sU + (c0 + 1) * R);
-#pragma unroll
-            for (int i = 0; i < RP; ++i) {
-              const uint64_t ua = u0[i];
-              cj[i] = fma2(e0, ua, cj[i]);
-              vj[i] = fma2(ua, we0, vj[i]);
-            }
-#pragma unroll
-            for (int i = 0; i < RP; ++i) {
-              const uint64_t ub = u1[i];
-              cj[i] = fma2(e1, ub, cj[i]);
-              vj[i] = fma2(ub, we1, vj[i]);
-            }
-            float t0, t1, w0, w1;
-            f2unpack(mul2(E2, E2), t0, t1);
-            f2unpack(w2, w0, w1);
-            err0 = __fmaf_rn(w0, t0, err0);
-            err0 = __fmaf_rn(w1, t1, err0);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if (i == wd) cw[i] = word;
-  }
-  reinterpret_cast<uint4*>(dcodes)[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-  reinterpret_cast<uint4*>(dcodes)[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-  if constexpr (ng == 4) {
-    uint2 sv;
-    sv.x = (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
-    sv.y = (uint32_t)__half_as_ushort(sh[2]) | ((uint32_t)__half_as_ushort(sh[3]) << 16);
-    *reinterpret_cast<uint2*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 8) = sv;
-  } else {
-    *reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 4) =
-        (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
-  }
-  tb[(is_key ? L.k_ids : L.v_ids) + tid] = (uint8_t)id;
-  {
-    uint8_t* dz = tb + (is_key ? L.k_zeros : L.v_zeros) + (int64_t)tid * L.zb;
-    dz[0] = (uint8_t)zbyte;
-    for (int b = 1; b < L.zb; ++b) dz[b] = 0;
-  }
-
-  // ---- 5. PSAC coefficients (Eq. 13, INT8 with a binary16 row scale) and
-  // the keep rule (Eq. 16), Keys only
-  if constexpr (R > 0) {
-    if (is_key) {
-      int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)tid * R);
-      __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma) + tid;
-      uint32_t cwd[R / 4];
-#pragma unroll
-      for (int i = 0; i < R / 4; ++i) cwd[i] = 0;
-      __half sgh_out = __ushort_as_half(0);
       if (psac) {
-        float c[R], v[R];
-#pragma unroll
-        for (int i = 0; i < RP; ++i) {
-          f2unpack(cj[i], c[2 * i], c[2 * i + 1]);
-          f2unpack(vj[i], v[2 * i], v[2 * i + 1]);
+        __nv_bfloat16* ut = reinterpret_cast<__nv_bfloat16*>(head + L.ut);
+        const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
+        for (int i = tid; i < R * 128; i += QNT) ut[i] = Uh[(size_t)(i % 128) * R + i / 128];  // U_r^T [r][d]
+      }
+    }
+
+    // ---- per-(head, side) setup: w, W_g, U (fp32), U^T W U, |U|_F^2, max w
+    if (pair != cur_pair) {
+      __syncthreads();  // the previous unit's last readers of these arrays are done
+      sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
+      if constexpr (R > 0) {
+        if (psac) {
+          const __nv_bfloat16* Uh = a.U + (size_t)h * 128 * R;
+          for (int i = tid; i < 128 * R; i += QNT) sU[i] = __bfloat162float(Uh[i]);  // [d][r]
         }
-        float amax = 0.0f;
+      }
+      __syncthreads();
+      if (tid < ng) {
+        float Wg = 0.0f;
+        for (int c = tid * GS; c < (tid + 1) * GS; ++c) Wg = __fadd_rn(Wg, sW[c]);
+        sMisc[tid] = Wg;
+      }
+      if constexpr (R > 0) {
+        if (psac) {
+          // U^T W U (any order; it enters only with its error bound): thread
+          // (j, k pair) accumulates two entries over the channels
+          for (int e = tid; e < R * RP; e += QNT) {
+            const int j = e / RP, kp = e % RP;
+            uint64_t acc = 0;
+            for (int c = 0; c < 128; ++c) {
+              const float uw = sU[c * R + j] * sW[c];
+              acc = fma2(f2pack(uw, uw), *reinterpret_cast<const uint64_t*>(sU + c * R + 2 * kp), acc);
+            }
+            *reinterpret_cast<uint64_t*>(sG + j * R + 2 * kp) = acc;
+          }
+          float u2 = 0.0f;
 #pragma unroll
-        for (int j = 0; j < R; ++j) amax = fmaxf(amax, fabsf(c[j]));
-        const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
-        const float sg = __half2float(sgh);
-        const float sinv = sg != 0.0f ? __frcp_rn(sg) : 0.0f;
-        float chat[R];
-        uint32_t tq[R / 4];
+          for (int j = 0; j < R; ++j) u2 = fmaf(sU[tid * R + j], sU[tid * R + j], u2);
+          float wm = sW[tid];
 #pragma unroll
-        for (int i = 0; i < R / 4; ++i) tq[i] = 0;
-#pragma unroll
-        for (int j = 0; j < R; ++j) {
-          const float qq = sg != 0.0f ? fminf(fmaxf(rintf(__fmul_rn(c[j], sinv)), -127.0f), 127.0f) : 0.0f;
-          tq[j >> 2] |= ((uint32_t)(int)qq & 0xFFu) << (8 * (j & 3));
-          chat[j] = __fmul_rn(qq, sg);
+          for (int off = 16; off; off >>= 1) {
+            u2 += __shfl_xor_sync(0xFFFFFFFFu, u2, off);
+            wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, off));
+          }
+          if (lane == 0) {
+            sMisc[8 + warp] = u2;
+            sMisc[12 + warp] = wm;
+          }
         }
-        bool keep = false;  // sigma == 0: chat = 0, so errq == err0 and the rule says no
-        if (sg != 0.0f) {
-          // errq - err0 = chat^T G chat - 2 chat.v with G = U^T W U
-          float quad = 0.0f, cv = 0.0f, cn2 = 0.0f, vn2 = 0.0f;
+      }
+      __syncthreads();
+      cur_pair = pair;
+    }
+    float Wg[4];
 #pragma unroll
-          for (int j = 0; j < R; ++j) {
-            float gj = 0.0f;
+    for (int gi = 0; gi < 4; ++gi) Wg[gi] = gi < ng ? sMisc[gi] : 0.0f;
+
+    // ---- the filter's record for this token, then the tile
+    uint32_t rec[8];
 #pragma unroll
-            for (int k = 0; k < R; ++k) gj = fmaf(sG[j * R + k], chat[k], gj);
-            quad = fmaf(chat[j], gj, quad);
-            cv = fmaf(chat[j], v[j], cv);
-            cn2 = fmaf(chat[j], chat[j], cn2);
-            vn2 = fmaf(v[j], v[j], vn2);
+    for (int i = 0; i < 8; ++i) rec[i] = 0;
+    uint32_t* dcodes = reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_codes : L.v_codes) + tid * 32);
+    if (!all_cand && valid) {
+      const uint4 r0 = ldg16(dcodes), r1 = ldg16(dcodes + 4);
+      rec[0] = r0.x; rec[1] = r0.y; rec[2] = r0.z; rec[3] = r0.w;
+      rec[4] = r1.x; rec[5] = r1.y; rec[6] = r1.z; rec[7] = r1.w;
+    }
+    if (tid == 0) *sRsCount = 0;  // the previous unit's list was last read before a barrier
+    const bool ok = mbar_wait(bar, ph);
+    ph ^= 1;
+    if (__syncthreads_or(!ok)) {
+      if (tid == 0) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_TIMEOUT);
+      break;
+    }
+
+    // ---- part A (reads the tile): candidates, QSAC, INT2 parameters, the
+    // channel pass
+    int id = 0;
+    const __nv_bfloat16* mr = tab;
+    float sc[4], inv[4], zf[4];
+    __half sh[4];
+    uint32_t zbyte = 0;
+    uint64_t cj[RP], vj[RP];
+#pragma unroll
+    for (int i = 0; i < RP; ++i) { cj[i] = 0; vj[i] = 0; }
+    float err0 = 0.0f;
+    uint32_t cw[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) cw[i] = 0;
+#pragma unroll
+    for (int gi = 0; gi < 4; ++gi) { sc[gi] = 0.0f; inv[gi] = 0.0f; zf[gi] = 0.0f; sh[gi] = __ushort_as_half(0); }
+
+    // ---- 1. candidates: the filter's decided top-M, or an exact rescoring
+    // of the band members (every centroid when the band was not listed).
+    // Rescoring is done by the whole CTA: each such token reserves a slice
+    // of the (token, centroid) list, every thread evaluates list entries,
+    // and the owner keeps the M smallest (dQ, j) of its slice.
+    int cand[kMaxFilterM];
+#pragma unroll
+    for (int s = 0; s < kMaxFilterM; ++s) cand[s] = 0;
+    bool rescore = false;
+    int rs_base = 0, rs_n = 0;
+    bool band = false;
+    if (valid && !all_cand) {
+      auto rb = [&](int i) -> int { return (int)((rec[i >> 2] >> (8 * (i & 3))) & 0xFFu); };
+      const int n = rb(0);
+      bool idsok = true;
+#pragma unroll
+      for (int i = 1; i <= kBand; ++i)
+        if (i <= n && rb(i) >= C) idsok = false;
+      if (n == Mc && idsok) {
+#pragma unroll
+        for (int s = 0; s < kMaxFilterM; ++s) cand[s] = rb(1 + s);
+      } else {
+        rescore = true;
+        band = n >= Mc && n <= kBand && idsok;  // a band holds at least M members
+        rs_n = band ? n : C;
+        rs_base = atomicAdd(sRsCount, rs_n);
+        if (rs_base + rs_n <= kRsCap) {
+          for (int m = 0; m < rs_n; ++m) {
+            int j = m;
+            if (band) {
+#pragma unroll
+              for (int i = 0; i < kBand; ++i)
+                if (i == m) j = rb(1 + i);
+            }
+            sRsPair[rs_base + m] = (uint16_t)((tid << 8) | j);
           }
-          float UF2 = 0.0f, wmax = 0.0f;
+        }
+      }
+    }
+    if (__syncthreads_or(rescore)) {
+      const int total = min(*sRsCount, kRsCap);
+      for (int q = tid; q < total; q += QNT) {
+        const int pr = sRsPair[q];
+        sRsDq[q] = exact_dq(sK, pr >> 8, tab + (size_t)(pr & 0xFF) * 128, sW);
+      }
+      __syncthreads();
+      if (rescore) {
+        float ev[kMaxFilterM];
+        int ej[kMaxFilterM];
 #pragma unroll
-          for (int i = 0; i < QNT / 32; ++i) {
-            UF2 += sMisc[8 + i];
-            wmax = fmaxf(wmax, sMisc[12 + i]);
+        for (int s = 0; s < kMaxFilterM; ++s) { ev[s] = INFINITY; ej[s] = 0x7FFFFFFF; }
+        float ek = INFINITY;
+        const bool listed = rs_base + rs_n <= kRsCap;
+        for (int m = 0; m < rs_n; ++m) {  // ascending j in both cases
+          float dq;
+          int j;
+          if (listed) {
+            j = sRsPair[rs_base + m] & 0xFF;
+            dq = sRsDq[rs_base + m];
+          } else {
+            j = m;
+            if (band) {
+              auto rb = [&](int i) -> int { return (int)((rec[i >> 2] >> (8 * (i & 3))) & 0xFFu); };
+#pragma unroll
+              for (int i = 0; i < kBand; ++i)
+                if (i == m) j = rb(1 + i);
+            }
+            dq = exact_dq(sK, tid, tab + (size_t)j * 128, sW);
           }
-          const float delta = fmaf(-2.0f, cv, quad);
-          const float eq = fabsf(err0 + delta);
-          const float Q = wmax * UF2 * cn2 * 1.0001f;
-          const float bound =
-              ldexpf(eq + err0 + Q + sqrtf(err0 * Q) + sqrtf(eq * Q) + sqrtf(cn2 * vn2), -14) + 1e-35f;
-          if (delta < -bound) {
-            keep = true;
-          } else if (!(delta > bound)) {
-            // too close to call: the sequential evaluation of both sums
-            float errq = 0.0f, e0 = 0.0f;
-#pragma unroll 1
-            for (int wd = 0; wd < 8; ++wd) {
-              const int gi = (wd * 16) / GS;
-              const float s = sel4(sc, gi), z = sel4(zf, gi);
-              uint32_t word = cw[0];
+          if (dq < ek) {
+            insert_top(ev, ej, Mc, dq, j);
+            ek = sel_at(ev, Mc - 1);
+          }
+        }
 #pragma unroll
-              for (int i = 1; i < 8; ++i)
-                if (i == wd) word = cw[i];
-#pragma unroll
-              for (int hc = 0; hc < 2; ++hc) {
-                const int ch = 2 * wd + hc;
-                const uint4 kv = lds16(sK + sw_off(128, tid, ch));
-                const uint4 mv = ldg16(mr + ch * 8);
-                const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                  const int c = ch * 8 + e;
-                  const float kf = __uint_as_float((e & 1) ? (kw[e >> 1] & 0xFFFF0000u) : (kw[e >> 1] << 16));
-                  const float mf = __uint_as_float((e & 1) ? (mw[e >> 1] & 0xFFFF0000u) : (mw[e >> 1] << 16));
-                  const int j16 = 8 * hc + e;
-                  const float q = (float)((word >> (16 * (j16 & 1) + 2 * (j16 >> 1))) & 3u);
-                  const float E = __fsub_rn(kf, __fadd_rn(mf, __fmul_rn(__fsub_rn(q, z), s)));
-                  float u = 0.0f;
-#pragma unroll
-                  for (int j = 0; j < R; ++j) u = __fmaf_rn(sU[c * R + j], chat[j], u);
-                  const float ep = __fsub_rn(E, u);
-                  errq = __fmaf_rn(sW[c], __fmul_rn(ep, ep), errq);
-                  e0 = __fmaf_rn(sW[c], __fmul_rn(E, E), e0);
-                }
+        for (int s = 0; s < kMaxFilterM; ++s) cand[s] = ej[s];
+      }
+    }
+
+    if (valid) {
+      // ---- 2. QSAC score (Eq. 10, 12) of each candidate, lowest (S, j); the
+      // group minima / maxima of the chosen residual feed the INT2 step.
+      // Candidates are scored QB at a time, channel blocks of 16 outermost, so
+      // that each block of the token row is read once per batch and the batch's
+      // centroid rows are in flight together (32-byte loads, whole sectors).
+      constexpr int QB = 4;
+      float bestS = INFINITY;
+      int bestj = 0x7FFFFFFF;
+      float bmn[4], bmx[4];
+    #pragma unroll
+      for (int gi = 0; gi < 4; ++gi) { bmn[gi] = 0.0f; bmx[gi] = 0.0f; }
+      const int ncand = all_cand ? C : Mc;
+      for (int m0 = 0; m0 < ncand; m0 += QB) {
+        const int nb = ncand - m0 < QB ? ncand - m0 : QB;
+        int jb[QB];
+    #pragma unroll
+        for (int b = 0; b < QB; ++b) {
+          const int m = m0 + b < ncand ? m0 + b : m0;
+          int j = m;
+          if (!all_cand) {
+    #pragma unroll
+            for (int s = 0; s < kMaxFilterM; ++s)
+              if (s == m) j = cand[s];
+          }
+          jb[b] = j;
+        }
+        float mx[QB][4], mn[QB][4];
+    #pragma unroll
+        for (int b = 0; b < QB; ++b)
+    #pragma unroll
+          for (int gi = 0; gi < 4; ++gi) { mx[b][gi] = -INFINITY; mn[b][gi] = INFINITY; }
+    #pragma unroll
+        for (int cc = 0; cc < 8; ++cc) {
+          const int gi = (cc * 16) / GS;
+          const uint4 ka = lds16(sK + sw_off(128, tid, 2 * cc)), kb = lds16(sK + sw_off(128, tid, 2 * cc + 1));
+          const uint32_t kw[8] = {ka.x, ka.y, ka.z, ka.w, kb.x, kb.y, kb.z, kb.w};
+          uint64_t k2[8];
+    #pragma unroll
+          for (int p = 0; p < 8; ++p) k2[p] = bf2_to_f2(kw[p]);
+    #pragma unroll
+          for (int b = 0; b < QB; ++b) {
+            if (b < nb) {
+              uint32_t mw[8];
+              ldg32(tab + (size_t)jb[b] * 128 + cc * 16, mw);
+              float x[16];
+    #pragma unroll
+              for (int p = 0; p < 8; ++p) f2unpack(sub2(k2[p], bf2_to_f2(mw[p])), x[2 * p], x[2 * p + 1]);
+    #pragma unroll
+              for (int e = 0; e < 16; e += 2) {
+                mx[b][gi] = fmax3f(mx[b][gi], x[e], x[e + 1]);
+                mn[b][gi] = fmin3(mn[b][gi], x[e], x[e + 1]);
               }
             }
-            keep = errq < e0;
           }
         }
-        if (keep) {
-#pragma unroll
-          for (int i = 0; i < R / 4; ++i) cwd[i] = tq[i];
-          sgh_out = sgh;
+    #pragma unroll
+        for (int b = 0; b < QB; ++b) {
+          if (b < nb) {
+            float Sc = 0.0f;
+    #pragma unroll
+            for (int gi = 0; gi < ng; ++gi) {
+              const float Rg = __fsub_rn(mx[b][gi], mn[b][gi]);
+              Sc = __fadd_rn(Sc, __fmul_rn(Wg[gi], __fmul_rn(Rg, Rg)));
+            }
+            const int j = jb[b];
+            if (Sc < bestS || (Sc == bestS && j < bestj)) {
+              bestS = Sc;
+              bestj = j;
+    #pragma unroll
+              for (int gi = 0; gi < 4; ++gi) { bmn[gi] = mn[b][gi]; bmx[gi] = mx[b][gi]; }
+            }
+          }
         }
       }
-      if constexpr (R == 8) {
-        *reinterpret_cast<uint2*>(coef) = make_uint2(cwd[0], cwd[1]);
-      } else {
-#pragma unroll
-        for (int i = 0; i < R / 16; ++i)
-          reinterpret_cast<uint4*>(coef)[i] = make_uint4(cwd[4 * i], cwd[4 * i + 1], cwd[4 * i + 2], cwd[4 * i + 3]);
+      id = bestj < C ? bestj : C - 1;
+      mr = tab + (size_t)id * 128;
+
+      // ---- 3. INT2 parameters (Eq. 1-2): range of the residual with 0 included
+    #pragma unroll
+      for (int gi = 0; gi < 4; ++gi) {
+        sc[gi] = 0.0f; inv[gi] = 0.0f; zf[gi] = 0.0f; sh[gi] = __ushort_as_half(0);
+        if (gi < ng) {
+          const float lo = fminf(0.0f, bmn[gi]), hi = fmaxf(0.0f, bmx[gi]);
+          sh[gi] = __float2half_ru(__fdiv_rn(__fsub_rn(hi, lo), 3.0f));
+          sc[gi] = __half2float(sh[gi]);
+          int zq = 0;
+          if (sc[gi] != 0.0f) {
+            inv[gi] = __frcp_rn(sc[gi]);
+            const int z = (int)rintf(__fmul_rn(-lo, inv[gi]));
+            zq = z < 0 ? 0 : (z > 3 ? 3 : z);
+          }
+          zf[gi] = (float)zq;
+          zbyte |= (uint32_t)zq << (2 * gi);
+        }
       }
-      *sig = sgh_out;
+
+      // ---- 4. one channel pass: INT2 codes; Keys with PSAC also E (Eq. 4, 13),
+      // c = U^T E, v = U^T (w o E) and err0 = sum_c w_c E_c^2, in channel order
+      const uint64_t MAG2 = f2pack(kMagic, kMagic);
+      uint32_t mwn[8];
+      ldg32(mr, mwn);
+    #pragma unroll 1
+      for (int wd = 0; wd < 8; ++wd) {
+        const int gi = (wd * 16) / GS;
+        const float s = sel4(sc, gi), iv = sel4(inv, gi), z = sel4(zf, gi);
+        const uint64_t S2 = f2pack(s, s), Z2 = f2pack(z, z);
+        uint32_t word = 0;
+        uint32_t mw8[8];
+    #pragma unroll
+        for (int i = 0; i < 8; ++i) mw8[i] = mwn[i];
+        if (wd < 7) ldg32(mr + (wd + 1) * 16, mwn);  // the next word's centroid chunk, one step ahead
+    #pragma unroll
+        for (int hc = 0; hc < 2; ++hc) {
+          const int ch = 2 * wd + hc;
+          const uint4 kv = lds16(sK + sw_off(128, tid, ch));
+          const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
+    #pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const uint64_t k2 = bf2_to_f2(kw[p]), m2 = bf2_to_f2(mw8[4 * hc + p]);
+            float x0, x1;
+            f2unpack(sub2(k2, m2), x0, x1);
+            // y = x * (1/s) rounded on its own (the scalar intrinsic is never fused
+            // into the following add), then rint(y) in both lanes
+            const uint64_t y2 = f2pack(__fmul_rn(x0, iv), __fmul_rn(x1, iv));
+            const uint64_t r2 = sub2(add2(y2, MAG2), MAG2);
+            float q0, q1;
+            f2unpack(add2(r2, Z2), q0, q1);
+            q0 = fminf(fmaxf(q0, 0.0f), 3.0f);
+            q1 = fminf(fmaxf(q1, 0.0f), 3.0f);
+            const uint32_t b0 = __float_as_uint(q0 + kTwo23) & 3u, b1 = __float_as_uint(q1 + kTwo23) & 3u;
+            word |= (b0 | (b1 << 16)) << (8 * hc + 2 * p);
+            if constexpr (R > 0) {
+              if (psac) {
+                // E = k - (mu + (q - z) s), then the channel pair's PSAC terms
+                const uint64_t dq2 = sub2(f2pack(q0, q1), Z2);
+                const uint64_t E2 = sub2(k2, add2(m2, mul2(dq2, S2)));
+                const int c0 = ch * 8 + 2 * p;
+                const uint64_t w2 = *reinterpret_cast<const uint64_t*>(sW + c0);
+                const uint64_t wE2 = mul2(w2, E2);
+                float E0, E1, wE0, wE1;
+                f2unpack(E2, E0, E1);
+                f2unpack(wE2, wE0, wE1);
+                const uint64_t e0 = f2pack(E0, E0), e1 = f2pack(E1, E1);
+                const uint64_t we0 = f2pack(wE0, wE0), we1 = f2pack(wE1, wE1);
+                const uint4* u0 = reinterpret_cast<const uint4*>(sU + c0 * R);
+                const uint4* u1 = reinterpret_cast<const uint4*>(sU + (c0 + 1) * R);
+    #pragma unroll
+                for (int i = 0; i < RP / 2; ++i) {
+                  const uint4 q = u0[i];
+                  const uint64_t ua = f2pack(__uint_as_float(q.x), __uint_as_float(q.y));
+                  const uint64_t ub = f2pack(__uint_as_float(q.z), __uint_as_float(q.w));
+                  cj[2 * i] = fma2(e0, ua, cj[2 * i]);
+                  vj[2 * i] = fma2(ua, we0, vj[2 * i]);
+                  cj[2 * i + 1] = fma2(e0, ub, cj[2 * i + 1]);
+                  vj[2 * i + 1] = fma2(ub, we0, vj[2 * i + 1]);
+                }
+    #pragma unroll
+                for (int i = 0; i < RP / 2; ++i) {
+                  const uint4 q = u1[i];
+                  const uint64_t ua = f2pack(__uint_as_float(q.x), __uint_as_float(q.y));
+                  const uint64_t ub = f2pack(__uint_as_float(q.z), __uint_as_float(q.w));
+                  cj[2 * i] = fma2(e1, ua, cj[2 * i]);
+                  vj[2 * i] = fma2(ua, we1, vj[2 * i]);
+                  cj[2 * i + 1] = fma2(e1, ub, cj[2 * i + 1]);
+                  vj[2 * i + 1] = fma2(ub, we1, vj[2 * i + 1]);
+                }
+                float t0, t1, w0, w1;
+                f2unpack(mul2(E2, E2), t0, t1);
+                f2unpack(w2, w0, w1);
+                err0 = __fmaf_rn(w0, t0, err0);
+                err0 = __fmaf_rn(w1, t1, err0);
+              }
+            }
+          }
+        }
+    #pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (i == wd) cw[i] = word;
+      }
+    }
+    // every read of the tile is done: refill it with the next unit's tokens
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0 && u + 1 < u1) issue_tile(u + 1);
+
+    // ---- part B: stores, PSAC
+    if (valid) {
+      reinterpret_cast<uint4*>(dcodes)[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+      reinterpret_cast<uint4*>(dcodes)[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+      if constexpr (ng == 4) {
+        uint2 sv;
+        sv.x = (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
+        sv.y = (uint32_t)__half_as_ushort(sh[2]) | ((uint32_t)__half_as_ushort(sh[3]) << 16);
+        *reinterpret_cast<uint2*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 8) = sv;
+      } else {
+        *reinterpret_cast<uint32_t*>(tb + (is_key ? L.k_scales : L.v_scales) + tid * 4) =
+            (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
+      }
+      tb[(is_key ? L.k_ids : L.v_ids) + tid] = (uint8_t)id;
+      {
+        uint8_t* dz = tb + (is_key ? L.k_zeros : L.v_zeros) + (int64_t)tid * L.zb;
+        dz[0] = (uint8_t)zbyte;
+        for (int b = 1; b < L.zb; ++b) dz[b] = 0;
+      }
+
+      // ---- 5. PSAC coefficients (Eq. 13, INT8 with a binary16 row scale) and
+      // the keep rule (Eq. 16), Keys only
+      if constexpr (R > 0) {
+        if (is_key) {
+          int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)tid * R);
+          __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma) + tid;
+          uint32_t cwd[R / 4];
+    #pragma unroll
+          for (int i = 0; i < R / 4; ++i) cwd[i] = 0;
+          __half sgh_out = __ushort_as_half(0);
+          if (psac) {
+            float c[R], v[R];
+    #pragma unroll
+            for (int i = 0; i < RP; ++i) {
+              f2unpack(cj[i], c[2 * i], c[2 * i + 1]);
+              f2unpack(vj[i], v[2 * i], v[2 * i + 1]);
+            }
+            float amax = 0.0f;
+    #pragma unroll
+            for (int j = 0; j < R; ++j) amax = fmaxf(amax, fabsf(c[j]));
+            const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
+            const float sg = __half2float(sgh);
+            const float sinv = sg != 0.0f ? __frcp_rn(sg) : 0.0f;
+            float chat[R];
+            uint32_t tq[R / 4];
+    #pragma unroll
+            for (int i = 0; i < R / 4; ++i) tq[i] = 0;
+    #pragma unroll
+            for (int j = 0; j < R; ++j) {
+              const float qq = sg != 0.0f ? fminf(fmaxf(rintf(__fmul_rn(c[j], sinv)), -127.0f), 127.0f) : 0.0f;
+              tq[j >> 2] |= ((uint32_t)(int)qq & 0xFFu) << (8 * (j & 3));
+              chat[j] = __fmul_rn(qq, sg);
+            }
+            bool keep = false;  // sigma == 0: chat = 0, so errq == err0 and the rule says no
+            if (sg != 0.0f) {
+              // errq - err0 = chat^T G chat - 2 chat.v with G = U^T W U
+              float quad = 0.0f, cv = 0.0f, cn2 = 0.0f, vn2 = 0.0f;
+    #pragma unroll
+              for (int j = 0; j < R; ++j) {
+                float gj = 0.0f;
+    #pragma unroll
+                for (int k = 0; k < R; ++k) gj = fmaf(sG[j * R + k], chat[k], gj);
+                quad = fmaf(chat[j], gj, quad);
+                cv = fmaf(chat[j], v[j], cv);
+                cn2 = fmaf(chat[j], chat[j], cn2);
+                vn2 = fmaf(v[j], v[j], vn2);
+              }
+              float UF2 = 0.0f, wmax = 0.0f;
+    #pragma unroll
+              for (int i = 0; i < QNT / 32; ++i) {
+                UF2 += sMisc[8 + i];
+                wmax = fmaxf(wmax, sMisc[12 + i]);
+              }
+              const float delta = fmaf(-2.0f, cv, quad);
+              const float eq = fabsf(err0 + delta);
+              const float Q = wmax * UF2 * cn2 * 1.0001f;
+              const float bound =
+                  ldexpf(eq + err0 + Q + sqrtf(err0 * Q) + sqrtf(eq * Q) + sqrtf(cn2 * vn2), -14) + 1e-35f;
+              if (delta < -bound) {
+                keep = true;
+              } else if (!(delta > bound)) {
+                // too close to call: the sequential evaluation of both sums
+                float errq = 0.0f, e0 = 0.0f;
+    #pragma unroll 1
+                for (int wd = 0; wd < 8; ++wd) {
+                  const int gi = (wd * 16) / GS;
+                  const float s = sel4(sc, gi), z = sel4(zf, gi);
+                  uint32_t word = cw[0];
+    #pragma unroll
+                  for (int i = 1; i < 8; ++i)
+                    if (i == wd) word = cw[i];
+    #pragma unroll
+                  for (int hc = 0; hc < 2; ++hc) {
+                    const int ch = 2 * wd + hc;
+                    const uint4 kv = ldg16(xr + ch * 8);
+                    const uint4 mv = ldg16(mr + ch * 8);
+                    const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w}, mw[4] = {mv.x, mv.y, mv.z, mv.w};
+    #pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                      const int c = ch * 8 + e;
+                      const float kf = __uint_as_float((e & 1) ? (kw[e >> 1] & 0xFFFF0000u) : (kw[e >> 1] << 16));
+                      const float mf = __uint_as_float((e & 1) ? (mw[e >> 1] & 0xFFFF0000u) : (mw[e >> 1] << 16));
+                      const int j16 = 8 * hc + e;
+                      const float q = (float)((word >> (16 * (j16 & 1) + 2 * (j16 >> 1))) & 3u);
+                      const float E = __fsub_rn(kf, __fadd_rn(mf, __fmul_rn(__fsub_rn(q, z), s)));
+                      float u = 0.0f;
+    #pragma unroll
+                      for (int j = 0; j < R; ++j) u = __fmaf_rn(sU[c * R + j], chat[j], u);
+                      const float ep = __fsub_rn(E, u);
+                      errq = __fmaf_rn(sW[c], __fmul_rn(ep, ep), errq);
+                      e0 = __fmaf_rn(sW[c], __fmul_rn(E, E), e0);
+                    }
+                  }
+                }
+                keep = errq < e0;
+              }
+            }
+            if (keep) {
+    #pragma unroll
+              for (int i = 0; i < R / 4; ++i) cwd[i] = tq[i];
+              sgh_out = sgh;
+            }
+          }
+          if constexpr (R == 8) {
+            *reinterpret_cast<uint2*>(coef) = make_uint2(cwd[0], cwd[1]);
+          } else {
+    #pragma unroll
+            for (int i = 0; i < R / 16; ++i)
+              reinterpret_cast<uint4*>(coef)[i] = make_uint4(cwd[4 * i], cwd[4 * i + 1], cwd[4 * i + 2], cwd[4 * i + 3]);
+          }
+          *sig = sgh_out;
+        }
+      }
     }
   }
 }
@@ -887,8 +1076,16 @@ cudaError_t launch_quant(const AppendArgs& a, const CUtensorMap& tk, const CUten
   constexpr int smem = QSmem<R>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(append_quant<R, GS>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)((a.N + 127) / 128), (unsigned)a.L.H, 2);
-  append_quant<R, GS><<<grid, QNT, smem, st>>>(a, tk, tv);
+  int dev = 0, nsm = 0, cps = 0;
+  e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&cps, append_quant<R, GS>, QNT, smem);
+  if (e != cudaSuccess) return e;
+  const int tiles = (int)((a.N + 127) / 128);
+  const int units = tiles * a.L.H * 2;
+  const int slots = nsm * (cps > 0 ? cps : 1);
+  const unsigned grid = (unsigned)(units < slots ? units : slots);  // persistent: one wave
+  append_quant<R, GS><<<grid, QNT, smem, st>>>(a, tk, tv, tiles, units, nsm, cps > 0 ? cps : 1);
   return cudaGetLastError();
 }
 template <int R>

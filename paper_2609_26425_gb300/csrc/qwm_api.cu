@@ -170,7 +170,10 @@ qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* c, const void* 
   if (!same_shape(cfg, &c->cfg)) return QWM_ERR_INVALID_ARG;
   if (N < 1) return QWM_ERR_INVALID_ARG;
   if (N > c->L.T) return QWM_ERR_CAPACITY;
-  if (!aligned16(k) || !aligned16(v) || !aligned16(k_centroids) || !aligned16(v_centroids)) return QWM_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v)) return QWM_ERR_INVALID_ARG;
+  // the centroid rows are read as whole 32-byte sectors
+  if ((reinterpret_cast<uintptr_t>(k_centroids) & 31u) || (reinterpret_cast<uintptr_t>(v_centroids) & 31u))
+    return QWM_ERR_INVALID_ARG;
   if ((w && (reinterpret_cast<uintptr_t>(w) & 3u)) || (U && !aligned16(U))) return QWM_ERR_INVALID_ARG;
   if (c->appended >= c->L.max_chunks && !c->sliding_window) return QWM_ERR_CAPACITY;
   int slot = (int)(c->appended % c->L.max_chunks);

@@ -243,6 +243,12 @@ def test_error_paths():
     with pytest.raises(qwm.QwmError) as e:  # no keys at all
         qwm.qwm_attend(cfg, empty, dev(k[:4]))
     assert e.value.status == 1
+    fresh = qwm.Cache(cfg, 100, 1)
+    buf = torch.zeros(H * 16 * 128 + 8, dtype=torch.bfloat16, device="cuda")
+    kc16 = buf[8:].view(H, 16, 128)  # 16-byte aligned, not 32: centroid rows are read as 32-byte sectors
+    with pytest.raises(qwm.QwmError) as e:
+        qwm.qwm_quantize_append(cfg, fresh, dev(k[:10]), dev(v[:10]), kc16, kc16)
+    assert e.value.status == 1
     out = qwm.qwm_attend(cfg, cache, dev(k[:0]))  # Nq = 0 is a no-op
     assert out.shape[0] == 0
     torch.cuda.synchronize()
