@@ -39,9 +39,6 @@
 //
 // M >= C skips the filter (every centroid is a candidate); 8 < M < C goes to
 // the generic kernel (append_generic.cu).
-#include <cuda.h>
-#include <cudaTypedefs.h>
-
 #include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
 
@@ -1043,34 +1040,6 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
 // ============================================================================
 // Host side
 // ============================================================================
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
-            cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
-    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }();
-  return fn;
-}
-
-// Tensor map over bf16 tokens x[N][H][128]: boxes of 64 channels x 1 head x
-// 128 tokens, 128-byte swizzle (the layout of one K-major operand block);
-// rows past N read as zeros.
-bool token_map(CUtensorMap* m, const void* x, int64_t N, int H) {
-  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[3] = {128, (cuuint64_t)H, (cuuint64_t)N};
-  cuuint64_t strides[2] = {256, (cuuint64_t)H * 256};
-  cuuint32_t box[3] = {64, 1, 128};
-  cuuint32_t es[3] = {1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(x), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int R, int GS>
 cudaError_t launch_quant(const AppendArgs& a, const CUtensorMap& tk, const CUtensorMap& tv, cudaStream_t st) {
   constexpr int smem = QSmem<R>::BYTES;
@@ -1098,7 +1067,8 @@ cudaError_t launch_quant_r(const AppendArgs& a, const CUtensorMap& tk, const CUt
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
   if (a.M > kMaxFilterM && a.M < a.L.C) return launch_append_generic(a, st);
   alignas(64) CUtensorMap tk, tv;
-  if (!token_map(&tk, a.k, a.N, a.L.H) || !token_map(&tv, a.v, a.N, a.L.H)) return cudaErrorInvalidValue;
+  if (!make_token_map(&tk, a.k, a.N, a.L.H, 128) || !make_token_map(&tv, a.v, a.N, a.L.H, 128))
+    return cudaErrorInvalidValue;
   if (a.M < a.L.C) {
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);

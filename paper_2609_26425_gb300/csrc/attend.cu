@@ -349,18 +349,24 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
         ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1));
         if (!ok) break;
         tc_fence_after();
-        float v[32];
+        // ---- row maximum: the four 32-column blocks of S_i, two loads per wait
+        float va[32], vb[32];
         float mt = -INFINITY;
 #pragma unroll
-        for (int cb = 0; cb < 4; ++cb) {
-          tmem_ld32(tS + cb * 32, v);
+        for (int cp = 0; cp < 2; ++cp) {
+          tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
           if (nvalid == 128) {
 #pragma unroll
-            for (int e = 0; e < 32; e += 2) mt = fmax3(mt, v[e], v[e + 1]);
+            for (int e = 0; e < 32; e += 2) {
+              mt = fmax3(mt, va[e], va[e + 1]);
+              mt = fmax3(mt, vb[e], vb[e + 1]);
+            }
           } else {
 #pragma unroll
-            for (int e = 0; e < 32; ++e)
-              if (cb * 32 + e < nvalid) mt = fmaxf(mt, v[e]);
+            for (int e = 0; e < 32; ++e) {
+              if (64 * cp + e < nvalid) mt = fmaxf(mt, va[e]);
+              if (64 * cp + 32 + e < nvalid) mt = fmaxf(mt, vb[e]);
+            }
           }
         }
         const float m_new = fmaxf(m_run, mt);
@@ -376,36 +382,53 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
         if (__any_sync(0xFFFFFFFFu, need) && jt > 0) {
 #pragma unroll
           for (int cb = 0; cb < 4; ++cb) {
-            tmem_ld32(tO + cb * 32, v);
+            tmem_ld32(tO + cb * 32, va);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] *= alpha;
-            tmem_st32(tO + cb * 32, v);
+            for (int e = 0; e < 32; ++e) va[e] *= alpha;
+            tmem_st32(tO + cb * 32, va);
           }
         }
+        // ---- P = exp2(s * scale * log2(e) - m) as f16 pairs (one MUFU op per
+        // pair), written over the S columns already read; the row sum adds
+        // exactly those f16 values, 32 at a time in a packed f16 tree (each
+        // partial <= 32 * 2^8, exact to 2^-11 relative), then in fp32.
         const float mb = m_run * sl2;
         const uint64_t SL = splat2(sl2), MB = splat2(-mb);
-        float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-#pragma unroll
-        for (int cb = 0; cb < 4; ++cb) {
-          tmem_ld32(tS + cb * 32, v);
-          uint32_t pk[16];
+        float lsum = 0.0f;
+        auto exp_block = [&](const float (&v)[32], uint32_t (&pk)[16], int col0, bool full) {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            // x = s * scale * log2(e) - m, exp2 of the f16 pair in one MUFU op;
-            // P is the f16 MMA operand and the row sum adds exactly those values.
             float x0 = v[e], x1 = v[e + 1];
             fma2(x0, x1, SL, MB);
-            if (nvalid < 128) {
-              if (cb * 32 + e >= nvalid) x0 = -INFINITY;
-              if (cb * 32 + e + 1 >= nvalid) x1 = -INFINITY;
+            if (!full) {
+              if (col0 + e >= nvalid) x0 = -INFINITY;
+              if (col0 + e + 1 >= nvalid) x1 = -INFINITY;
             }
-            const uint32_t p2 = ex2_f16x2(pack_f16(x0, x1));
-            ls[(e >> 1) & 3] = add_f16lo(add_f16hi(ls[(e >> 1) & 3], p2), p2);
-            pk[e >> 1] = p2;
+            pk[e >> 1] = ex2_f16x2(pack_f16(x0, x1));
           }
-          tmem_st16(tS + cb * 16, pk);  // P (f16 pairs) over the columns already read
+        };
+        auto sum_block = [&](const uint32_t (&pk)[16]) -> float {
+          __half2 t8[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) t8[k] = __hadd2(u2h(pk[2 * k]), u2h(pk[2 * k + 1]));
+#pragma unroll
+          for (int k = 0; k < 4; ++k) t8[k] = __hadd2(t8[2 * k], t8[2 * k + 1]);
+          t8[0] = __hadd2(t8[0], t8[1]);
+          t8[2] = __hadd2(t8[2], t8[3]);
+          const float2 f = __half22float2(__hadd2(t8[0], t8[2]));
+          return f.x + f.y;
+        };
+#pragma unroll
+        for (int cp = 0; cp < 2; ++cp) {
+          tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
+          uint32_t pk[16];
+          exp_block(va, pk, 64 * cp, nvalid == 128);
+          tmem_st16(tS + 32 * cp, pk);  // P of columns 64cp..64cp+31 over columns already read
+          lsum += sum_block(pk);
+          exp_block(vb, pk, 64 * cp + 32, nvalid == 128);
+          tmem_st16(tS + 32 * cp + 16, pk);
+          lsum += sum_block(pk);
         }
-        const float lsum = (ls[0] + ls[1]) + (ls[2] + ls[3]);
         tmem_wait_st();
         l_run += lsum;
         tc_fence_before();

@@ -3,6 +3,7 @@
 // (tcgen05, mbarrier, bulk copies).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -71,6 +72,15 @@ inline Layout make_layout(const qwm_config& c, int64_t T, int32_t max_chunks) {
 __host__ __device__ inline int64_t head_offset(const Layout& L, int slot, int h) {
   return kHeaderBytes + (int64_t)slot * L.slot_bytes + kSlotMetaBytes + (int64_t)h * L.head_bytes;
 }
+
+// ----------------------------------------------------------------------------
+// TMA tensor maps (host, qwm_api.cu).
+// Tokens x[N][H][128] (bf16): boxes of 64 channels x 1 head x box_rows tokens,
+// 128-byte swizzle; rows past N read as zeros.
+bool make_token_map(CUtensorMap* m, const void* x, int64_t N, int H, int box_rows);
+// The cache buffer as rows of 256 bytes (128 binary16 values): boxes of 64
+// values x 1 row, 128-byte swizzle, for tile::gather4 loads of centroid rows.
+bool make_row_map(CUtensorMap* m, const void* base, int64_t rows);
 
 // ----------------------------------------------------------------------------
 // Kernel launch entry points (defined in the .cu files).
