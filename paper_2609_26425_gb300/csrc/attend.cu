@@ -513,11 +513,14 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
       uint8_t* dst = sm + (isK ? OFF_K : OFF_V) + st * 2 * BLK;
       const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
       const uint8_t* tab = cur.U.hb ? cur.U.hb + (isK ? L.ktab : L.vtab) : nullptr;
+      const bool psac_lane = isK && cur.U.psac && q * 8 < r;
 #pragma unroll
       for (int rd = 0; rd < 2; ++rd) {
         uint32_t mv[2][2][8];  // [pass][slice][words]
         uint32_t cwv[2][2];
         uint32_t scv[2][2];
+        uint2 cfv[2];          // PSAC INT8 codes 8q..8q+7 of the row (Keys)
+        uint32_t sgv[2];       // PSAC row scale (binary16 bits)
 #pragma unroll
         for (int pp = 0; pp < 2; ++pp) {
           const int p = 2 * rd + pp;
@@ -529,8 +532,14 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
             cwv[pp][sl] = 0u;
             scv[pp][sl] = 0u;
           }
+          cfv[pp] = make_uint2(0u, 0u);
+          sgv[pp] = 0u;
           if (row < nv) {
             if (tb) {
+              if (psac_lane) {  // the row's PSAC codes ride in the same round of loads
+                cfv[pp] = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)row * r + q * 8));
+                sgv[pp] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + row * 2));
+              }
               const uint8_t* mu = tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256;
               ldg32B(mu + 32 * q, mv[pp][0]);
               ldg32B(mu + 128 + 32 * q, mv[pp][1]);
@@ -581,26 +590,25 @@ __global__ void __launch_bounds__(NT, 1) attend_kernel(const AttendArgs a, const
             st_chunk(dst, row, c0, make_uint4(ow[0], ow[1], ow[2], ow[3]));
             st_chunk(dst, row, c0 + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]));
           }
-        }
-      }
-      if (isK && cur.U.psac && q * 8 < rpad) {
-        // C_hat = t * sigma, chunk q of the PSAC columns of each of the 4 rows
-        uint8_t* sC = sm + OFF_C;
+          if (isK && cur.U.psac && q * 8 < rpad) {
+            // C_hat = t * sigma (Eq. 16), PSAC columns 8q..8q+7 of the row, in
+            // f16: byte b of an INT8 code t becomes the f16 1024 + (t + 128)
+            // (its byte XOR 0x80 under exponent bits 0x64), minus 1152 gives t
+            // exactly, and one f16 multiply rounds t * sigma once.
+            uint32_t w4[4] = {0u, 0u, 0u, 0u};
+            if (tb && row < nv && q * 8 < r) {
+              const __half2 sg2 = u2h(sgv[pp] | (sgv[pp] << 16));
+              const __half2 off2 = u2h(0x64806480u);  // (1152, 1152)
+              const uint32_t cwd[2] = {cfv[pp].x ^ 0x80808080u, cfv[pp].y ^ 0x80808080u};
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const int row = wrow + 8 * p;
-          uint32_t w4[4] = {0u, 0u, 0u, 0u};
-          if (row < nv && q * 8 < r) {
-            const float sg = __half2float(*reinterpret_cast<const __half*>(tb + L.k_sigma + row * 2));
-            const uint2 cw = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)row * r + q * 8));
-            const uint32_t cwd[2] = {cw.x, cw.y};
-#pragma unroll
-            for (int q2 = 0; q2 < 4; ++q2) {
-              const uint32_t wd = cwd[q2 >> 1];
-              w4[q2] = pack_f16((float)(int8_t)(wd >> (16 * (q2 & 1))) * sg, (float)(int8_t)(wd >> (16 * (q2 & 1) + 8)) * sg);
+              for (int q2 = 0; q2 < 4; ++q2) {
+                const uint32_t b0 = 2 * (q2 & 1);
+                const uint32_t t2 = __byte_perm(cwd[q2 >> 1], 0x64646464u, b0 | (4u << 4) | ((b0 + 1) << 8) | (4u << 12));
+                w4[q2] = h2u(__hmul2(__hsub2(u2h(t2), off2), sg2));
+              }
             }
+            st_chunk(sm + OFF_C, row, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]));
           }
-          st_chunk(sC, row, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]));
         }
       }
       fence_proxy_async_smem();
