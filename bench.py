@@ -51,6 +51,28 @@ def workload_numbers(wl):
             "k_bytes_per_token_head": k_tok, "v_bytes_per_token_head": v_tok}
 
 
+def attend_traffic():
+    """DRAM bytes per attend launch from the committed ncu summary, or None when
+    the kernel source has changed since those counters were taken."""
+    import hashlib
+    prof = os.path.join(ROOT, "profiles", "attend_kernel_wan14b_layer.md")
+    src = os.path.join(ROOT, "paper_2609_26425_gb300", "csrc", "attend.cu")
+    try:
+        fields = {}
+        with open(prof) as f:
+            for line in f:
+                if ":" in line and line.split(":")[0] in ("traffic_bytes_per_launch", "source_sha256"):
+                    k, v = line.split(":", 1)
+                    fields[k.strip()] = v.strip()
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()
+        if fields.get("source_sha256") == digest:
+            return int(fields["traffic_bytes_per_launch"])
+    except (OSError, ValueError, KeyError):
+        pass
+    return None
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -269,7 +291,7 @@ def run_gpu(args, wl, rank, world):
                    "algorithmic_bytes": nums["append_bytes"]},
         "roofline": {"bound": "tensor", "kernel": "attend_kernel", "achieved": round(att_tflops, 2),
                      "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s",
-                     "frac": round(att_tflops / pk["bf16_tflops_sustained"], 4), "traffic": None,
+                     "frac": round(att_tflops / pk["bf16_tflops_sustained"], 4), "traffic": attend_traffic(),
                      "peak_src": pk["src"] + " sustained bf16"},
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         # attend: one kernel; append: the candidate filter and the quantize kernel
