@@ -286,16 +286,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         // ---- row maximum: the four 32-column blocks of S_i, two loads per wait
         float va[32], vb[32];
         float mt = -INFINITY;
+        if (nvalid == 128) {  // the TMEM loads reduce the columns they read
+          float m0, m1, m2, m3;
+          tmem_max32x2(tS, tS + 32, m0, m1);
+          tmem_max32x2(tS + 64, tS + 96, m2, m3);
+          mt = fmax3(fmaxf(m0, m1), m2, m3);
+        } else {
 #pragma unroll
-        for (int cp = 0; cp < 2; ++cp) {
-          tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
-          if (nvalid == 128) {
-#pragma unroll
-            for (int e = 0; e < 32; e += 2) {
-              mt = fmax3(mt, va[e], va[e + 1]);
-              mt = fmax3(mt, vb[e], vb[e + 1]);
-            }
-          } else {
+          for (int cp = 0; cp < 2; ++cp) {
+            tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
               if (64 * cp + e < nvalid) mt = fmaxf(mt, va[e]);
