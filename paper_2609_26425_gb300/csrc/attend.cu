@@ -292,7 +292,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           tmem_max32x2(tS + 64, tS + 96, m2, m3);
           mt = fmax3(fmaxf(m0, m1), m2, m3);
         } else {
-#pragma unroll
+#pragma unroll 1
           for (int cp = 0; cp < 2; ++cp) {
             tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
 #pragma unroll
@@ -313,7 +313,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         // S_i of this tile completing implies the previous P_i V MMA is done,
         // so O_i can be rescaled here.
         if (__any_sync(0xFFFFFFFFu, need) && jt > 0) {
-#pragma unroll
+#pragma unroll 1
           for (int cb = 0; cb < 4; ++cb) {
             tmem_ld32(tO + cb * 32, va);
 #pragma unroll
@@ -351,7 +351,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           const float2 f = __half22float2(__hadd2(t8[0], t8[2]));
           return f.x + f.y;
         };
-#pragma unroll
+#pragma unroll 1
         for (int cp = 0; cp < 2; ++cp) {
           tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
           uint32_t pk[16];
@@ -445,74 +445,65 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
       const uint8_t* tab = cur.U.hb ? cur.U.hb + L.ktab : nullptr;
       const bool psac_lane = cur.U.psac && q * 8 < r;
-      uint32_t mv[2][2][8];  // [pass][slice][words]
-      uint32_t cwv[2][2];
-      uint32_t scv[2][2];
-      uint2 cfv[2];          // PSAC INT8 codes 8q..8q+7 of the row
-      uint32_t sgv[2];       // PSAC row scale (binary16 bits)
-#pragma unroll
+      // One row per pass (loads, then its reconstruction); the pass loop is
+      // kept rolled so that the four roles' hot loops stay small enough for
+      // the instruction caches.
+#pragma unroll 1
       for (int p = 0; p < 2; ++p) {
         const int lr = wrow + 8 * p, trw = tro + lr;
+        const bool rv = trw < nv;
+        uint32_t mv[2][8];  // [slice][words]
+        uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
+        uint2 cfv = make_uint2(0u, 0u);  // PSAC INT8 codes 8q..8q+7 of the row
+        uint32_t sgv = 0u;               // PSAC row scale (binary16 bits)
 #pragma unroll
-        for (int sl = 0; sl < 2; ++sl) {
+        for (int sl = 0; sl < 2; ++sl)
 #pragma unroll
-          for (int e = 0; e < 8; ++e) mv[p][sl][e] = 0u;
-          cwv[p][sl] = 0u;
-          scv[p][sl] = 0u;
-        }
-        cfv[p] = make_uint2(0u, 0u);
-        sgv[p] = 0u;
-        if (trw < nv) {
+          for (int e = 0; e < 8; ++e) mv[sl][e] = 0u;
+        if (rv) {
           if (tb) {
             const uint8_t* mu = tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256;
-            ldg32B(mu + 32 * q, mv[p][0]);
-            ldg32B(mu + 128 + 32 * q, mv[p][1]);
+            ldg32B(mu + 32 * q, mv[0]);
+            ldg32B(mu + 128 + 32 * q, mv[1]);
             const uint8_t* cp = tb + L.k_codes + trw * 32;
-            cwv[p][0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
-            cwv[p][1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
+            cwv[0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
+            cwv[1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
             const unsigned short* sp = reinterpret_cast<const unsigned short*>(tb + L.k_scales + (int64_t)trw * L.ng * 2);
-            scv[p][0] = __ldg(sp + ((16 * q) >> gshift));
-            scv[p][1] = __ldg(sp + ((64 + 16 * q) >> gshift));
+            scv[0] = __ldg(sp + ((16 * q) >> gshift));
+            scv[1] = __ldg(sp + ((64 + 16 * q) >> gshift));
             if (psac_lane) {
-              cfv[p] = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
-              sgv[p] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
+              cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
+              sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
             }
           } else {
             const __nv_bfloat16* src = a.kcur + ((size_t)(cur.tl * 128 + trw) * H + h) * 128;
-            const uint4 v0 = ldg16(src + 16 * q), v1 = ldg16(src + 16 * q + 8);
-            const uint4 v2 = ldg16(src + 64 + 16 * q), v3 = ldg16(src + 64 + 16 * q + 8);
-            const uint4 f0 = bf16x8_to_f16x8(v0), f1 = bf16x8_to_f16x8(v1);
-            const uint4 f2 = bf16x8_to_f16x8(v2), f3 = bf16x8_to_f16x8(v3);
-            mv[p][0][0] = f0.x; mv[p][0][1] = f0.y; mv[p][0][2] = f0.z; mv[p][0][3] = f0.w;
-            mv[p][0][4] = f1.x; mv[p][0][5] = f1.y; mv[p][0][6] = f1.z; mv[p][0][7] = f1.w;
-            mv[p][1][0] = f2.x; mv[p][1][1] = f2.y; mv[p][1][2] = f2.z; mv[p][1][3] = f2.w;
-            mv[p][1][4] = f3.x; mv[p][1][5] = f3.y; mv[p][1][6] = f3.z; mv[p][1][7] = f3.w;
+#pragma unroll
+            for (int sl = 0; sl < 2; ++sl) {
+              const uint4 f0 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q));
+              const uint4 f1 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q + 8));
+              mv[sl][0] = f0.x; mv[sl][1] = f0.y; mv[sl][2] = f0.z; mv[sl][3] = f0.w;
+              mv[sl][4] = f1.x; mv[sl][5] = f1.y; mv[sl][6] = f1.z; mv[sl][7] = f1.w;
+            }
           }
         }
-      }
-#pragma unroll
-      for (int p = 0; p < 2; ++p) {
-        const int lr = wrow + 8 * p, trw = tro + lr;
+        const bool deq = tb && rv;
         const uint32_t zbyte = (idc >> (16 + 8 * p)) & 0xFFu;
 #pragma unroll
         for (int sl = 0; sl < 2; ++sl) {
           const int c0 = 8 * sl + 2 * q;  // first of the two chunks of this slice
+          // f16 pairs mu + (q - z) s; a row of the active chunk (or a padding
+          // row) passes through with s = 0 and z = q.
+          const int g = (64 * sl + 16 * q) >> gshift;
+          const uint32_t sb = deq ? scv[sl] : 0u;
+          const __half2 s2 = u2h(sb | (sb << 16));
+          const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
+          const __half2 z2 = u2h(zz | (zz << 16));
+          const uint32_t word = cwv[sl];
           uint32_t ow[8];
-          if (tb && trw < nv) {
-            const int g = (64 * sl + 16 * q) >> gshift;
-            const uint32_t sb = scv[p][sl];
-            const __half2 s2 = u2h(sb | (sb << 16));
-            const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
-            const __half2 z2 = u2h(zz | (zz << 16));
-            const uint32_t word = cwv[p][sl];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {  // channel pairs (2k, 2k+1) of the 16-channel word
-              const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
-              ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[p][sl][k])));
-            }
-          } else {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) ow[k] = mv[p][sl][k];
+          for (int k = 0; k < 8; ++k) {  // channel pairs (2k, 2k+1) of the 16-channel word
+            const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+            ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[sl][k])));
           }
           st_chunk(dst, lr, c0, make_uint4(ow[0], ow[1], ow[2], ow[3]), 64);
           st_chunk(dst, lr, c0 + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]), 64);
@@ -521,18 +512,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           // C_hat = t * sigma (Eq. 16), PSAC columns 8q..8q+7 of the row, in
           // f16: byte b of an INT8 code t becomes the f16 1024 + (t + 128)
           // (its byte XOR 0x80 under exponent bits 0x64), minus 1152 gives t
-          // exactly, and one f16 multiply rounds t * sigma once.
-          uint32_t w4[4] = {0u, 0u, 0u, 0u};
-          if (tb && trw < nv && q * 8 < r) {
-            const __half2 sg2 = u2h(sgv[p] | (sgv[p] << 16));
-            const __half2 off2 = u2h(0x64806480u);  // (1152, 1152)
-            const uint32_t cwd[2] = {cfv[p].x ^ 0x80808080u, cfv[p].y ^ 0x80808080u};
+          // exactly, and one f16 multiply rounds t * sigma once.  Lanes past
+          // r and padding rows hold zero codes and scale: zero columns.
+          const __half2 sg2 = u2h(sgv | (sgv << 16));
+          const __half2 off2 = u2h(0x64806480u);  // (1152, 1152)
+          const uint32_t cwd[2] = {cfv.x ^ 0x80808080u, cfv.y ^ 0x80808080u};
+          uint32_t w4[4];
 #pragma unroll
-            for (int q2 = 0; q2 < 4; ++q2) {
-              const uint32_t b0 = 2 * (q2 & 1);
-              const uint32_t t2 = __byte_perm(cwd[q2 >> 1], 0x64646464u, b0 | (4u << 4) | ((b0 + 1) << 8) | (4u << 12));
-              w4[q2] = h2u(__hmul2(__hsub2(u2h(t2), off2), sg2));
-            }
+          for (int q2 = 0; q2 < 4; ++q2) {
+            const uint32_t b0 = 2 * (q2 & 1);
+            const uint32_t t2 = __byte_perm(cwd[q2 >> 1], 0x64646464u, b0 | (4u << 4) | ((b0 + 1) << 8) | (4u << 12));
+            w4[q2] = h2u(__hmul2(__hsub2(u2h(t2), off2), sg2));
           }
           st_chunk(sm + OFF_C, lr, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]), 64);
         }
@@ -587,19 +577,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
       const uint8_t* tab = cur.U.hb ? cur.U.hb + L.vtab : nullptr;
       const int g = (16 * c16) >> gshift;
-#pragma unroll
+#pragma unroll 1
       for (int rd = 0; rd < 2; ++rd) {
         uint32_t mv[2][8];
-        uint32_t cwv[2];
-        uint32_t scv[2];
+        uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
 #pragma unroll
         for (int pp = 0; pp < 2; ++pp) {
           const int p = 2 * rd + pp;
           const int row = wrow + 8 * p;
 #pragma unroll
           for (int e = 0; e < 8; ++e) mv[pp][e] = 0u;
-          cwv[pp] = 0u;
-          scv[pp] = 0u;
           if (row < nv) {
             if (tb) {
               ldg32B(tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256 + 32 * c16, mv[pp]);
@@ -617,22 +604,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         for (int pp = 0; pp < 2; ++pp) {
           const int p = 2 * rd + pp;
           const int row = wrow + 8 * p;
+          // mu + (q - z) s; active-chunk and padding rows pass through with
+          // s = 0 and zero codes and zero-points (the ids word is 0 there).
+          const uint32_t zbyte = (uint32_t)((idc >> (32 + 8 * p)) & 0xFFu);
+          const uint32_t sb = scv[pp];
+          const __half2 s2 = u2h(sb | (sb << 16));
+          const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
+          const __half2 z2 = u2h(zz | (zz << 16));
+          const uint32_t word = cwv[pp];
           uint32_t ow[8];
-          if (tb && row < nv) {
-            const uint32_t zbyte = (uint32_t)((idc >> (32 + 8 * p)) & 0xFFu);
-            const uint32_t sb = scv[pp];
-            const __half2 s2 = u2h(sb | (sb << 16));
-            const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
-            const __half2 z2 = u2h(zz | (zz << 16));
-            const uint32_t word = cwv[pp];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
-              ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[pp][k])));
-            }
-          } else {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) ow[k] = mv[pp][k];
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+            ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[pp][k])));
           }
           st_chunk(dst, row, 2 * q, make_uint4(ow[0], ow[1], ow[2], ow[3]));
           st_chunk(dst, row, 2 * q + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]));
