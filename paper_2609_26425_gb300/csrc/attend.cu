@@ -13,16 +13,19 @@
 //   warps 0-3, 4-7   softmax of Q tile 0 / 1: thread = query row; reads its
 //                    logit row S_i from TMEM, keeps the running max and sum,
 //                    writes P_i as f16 back into the same TMEM columns, and
-//                    at chunk boundaries computes Q U_r of the next chunk
-//                    (Sec. 4.2 Eq. 17) into the extra Q operand columns;
+//                    at chunk boundaries moves Q U_r of the next chunk
+//                    (Sec. 4.2 Eq. 17; computed by the tensor cores into
+//                    spare S_i columns) into the extra Q operand columns;
 //   warps 8-11       rebuild this CTA's 64 keys of K_hat0 = mu_id + s (q - z)
 //                    (Sec. 2 Eq. 4) of each 128-key tile into a 2-stage
 //                    shared-memory ring, plus their r PSAC columns
-//                    C_hat = t * sigma (Eq. 16);
+//                    C_hat = t * sigma (Eq. 16), and at a chunk's first tile
+//                    its U_r^T as the B operand of the Q U_r MMA;
 //   warps 12-15      rebuild this CTA's 64 channels of V_hat (same
 //                    reconstruction, no PSAC) for all 128 keys;
 //   warp 16          allocates the pair's TMEM; in the leader, one thread
-//                    issues every MMA: S_i = [Q_i | Q_i U_r] [K_hat0 | C_hat]^T
+//                    issues every MMA: Q_i U_r once per chunk,
+//                    S_i = [Q_i | Q_i U_r] [K_hat0 | C_hat]^T
 //                    (the PSAC logit term rides along as extra reduction
 //                    columns) and O_i += P_i V_hat with P_i read straight from
 //                    TMEM.
@@ -58,9 +61,12 @@ constexpr int OFF_QU = 4 * BLK;          // Q_i U_r at columns [i*rpad, (i+1)*rp
 constexpr int OFF_K = 5 * BLK;           // this CTA's 64 keys of K_hat0: stage s, block kb at (2s + kb) * HBLK
 constexpr int OFF_C = OFF_K + 4 * HBLK;  // their C_hat (64 rows), stage s at columns [s*rpad, (s+1)*rpad)
 constexpr int OFF_V = OFF_C + HBLK;      // this CTA's 64 channels of V_hat (128 keys), stage s at s * BLK
-constexpr int OFF_BAR = OFF_V + 2 * BLK;
+constexpr int OFF_U = OFF_V + 2 * BLK;    // U_r^T operand of the Q U_r MMA: chunk parity p, block kb at (2p + kb) * 4 KB
+constexpr int UBLK = 4096;                 // 32 rows x 128 bytes
+constexpr int OFF_BAR = OFF_U + 4 * UBLK;
 enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_PFULL = 10, B_QU = 12, B_OFINAL = 14,
-       NBAR = 15 };
+       B_QUMMA = 15, NBAR = 17 };
+static_assert(NBAR * 8 + 12 <= 256, "barrier area");
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;  // + alignment slack
 
 // 8 f16 (16 bytes) of row `row`, chunk `ch` (columns 8ch..8ch+7) into a run of
@@ -159,46 +165,18 @@ struct TileCursor {
   __device__ __forceinline__ int nvalid() const { return min(128, U.ntok - tl * 128); }
 };
 
-// Q_i U_r of one query row (fp32 sums of bf16 products), as f16 into the
-// shared Q U_r block at columns [i*rpad, i*rpad + rpad).
-__device__ __forceinline__ void write_qu(uint8_t* sQU, int i, int row, bool qvalid, const __nv_bfloat16* qrow,
-                                         const uint8_t* ut, int r, int rpad) {
-  float acc[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) acc[j] = 0.0f;
-  if (qvalid) {
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 qv = ldg16(qrow + ch * 8);
-      const uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
-      float qf[8];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        qf[2 * e] = __uint_as_float(qw[e] << 16);
-        qf[2 * e + 1] = __uint_as_float(qw[e] & 0xFFFF0000u);
-      }
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        if (j < r) {
-          const uint4 uv = ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2);
-          const uint32_t uw[4] = {uv.x, uv.y, uv.z, uv.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            acc[j] = fmaf(qf[2 * e], __uint_as_float(uw[e] << 16), acc[j]);
-            acc[j] = fmaf(qf[2 * e + 1], __uint_as_float(uw[e] & 0xFFFF0000u), acc[j]);
-          }
-        }
-      }
-    }
-  }
+// Q_i U_r of one query row, computed by the tensor cores into TMEM columns
+// [64, 64 + rpad) of S_i, as f16 into the shared Q U_r block at columns
+// [i*rpad, (i+1)*rpad) (the A operand of the PSAC reduction columns).
+__device__ __forceinline__ void qu_to_smem(uint8_t* sQU, int i, int row, uint32_t tqu, int rpad) {
+  float v[32];
+  tmem_ld32(tqu, v);
 #pragma unroll
   for (int c2 = 0; c2 < 4; ++c2) {
     if (c2 * 8 < rpad) {
       uint32_t w4[4];
 #pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const int j = c2 * 8 + 2 * p;
-        w4[p] = pack_f16(j < r ? acc[j] : 0.0f, j + 1 < r ? acc[j + 1] : 0.0f);
-      }
+      for (int p = 0; p < 4; ++p) w4[p] = pack_f16(v[c2 * 8 + 2 * p], v[c2 * 8 + 2 * p + 1]);
       st_chunk(sQU, row, (i * rpad) / 8 + c2, make_uint4(w4[0], w4[1], w4[2], w4[3]));
     }
   }
@@ -240,6 +218,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       mbar_init(bar(B_QU + s), 8);
     }
     mbar_init(bar(B_OFINAL), 1);
+    mbar_init(bar(B_QUMMA), 1);         // Q_i U_r MMA commit, both CTAs
+    mbar_init(bar(B_QUMMA + 1), 1);
     *s_err = 0;
     fence_mbar_init();
   }
@@ -264,17 +244,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     uint8_t* sQi = sm + OFF_Q + i * 2 * BLK;
     if (qvalid) copy_row(sQi, row, qrow);
     else zero_row(sQi, row, 0, 16);
-    if (n_units > 0) {
-      const Unit u0 = unit_at(a, S, 0, h);
-      if (u0.psac) write_qu(sm + OFF_QU, i, row, qvalid, qrow, u0.hb + L.ut, r, rpad);
-    }
     fence_proxy_async_smem();
-    arrive_leader(B_QU + i);
+    arrive_leader(B_QU + i);  // Q_i is in place
+    // Q_i U_r of each chunk that carries PSAC columns: the MMA thread computes
+    // it into columns 64.. of S_i (free while S_i is not in use); this group
+    // moves it into the shared A operand of the extra reduction columns.
+    uint32_t qum = 0;  // completed Q_i U_r MMAs
+    auto take_qu = [&]() -> bool {
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1))) return false;
+      ++qum;
+      tc_fence_after();
+      qu_to_smem(sm + OFF_QU, i, row, tS + 64, rpad);
+      tc_fence_before();
+      fence_proxy_async_smem();
+      arrive_leader(B_QU + i);
+      return true;
+    };
 
     const float sl2 = a.sm_scale * 1.4426950408889634f;
     float m_run = -INFINITY, l_run = 0.0f;
     uint32_t jt = 0;
     bool ok = true;
+    if (n_units > 0 && unit_at(a, S, 0, h).psac) ok = take_qu();
     for (int u = 0; u < n_units && ok; ++u) {
       const Unit U = unit_at(a, S, u, h);
       const int ntiles = (U.ntok + 127) / 128;
@@ -367,15 +358,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         tc_fence_before();
         arrive_leader(B_PFULL + i);
       }
-      if (ok && u + 1 < n_units) {
-        const Unit Un = unit_at(a, S, u + 1, h);
-        if (Un.psac) {
-          // S_i of this chunk's last tile has completed: the Q U_r columns are free.
-          write_qu(sm + OFF_QU, i, row, qvalid, qrow, Un.hb + L.ut, r, rpad);
-          fence_proxy_async_smem();
-          arrive_leader(B_QU + i);
-        }
-      }
+      if (ok && u + 1 < n_units && unit_at(a, S, u + 1, h).psac) ok = take_qu();
     }
     if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFINAL), 0));
     if (ok) {
@@ -429,11 +412,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     uint32_t idn = load_ids(cur);
     uint32_t jt = 0;
     bool ok = true;
+    const int kt = tid - 32 * 8;  // 0..127
+    if (rank == 1)  // the follower's half of the U_r^T operand (rows 32..63 of N = 64) stays zero
+      for (int idx = kt; idx < 4 * UBLK / 16; idx += 128)
+        *reinterpret_cast<uint4*>(sm + OFF_U + 16 * idx) = make_uint4(0u, 0u, 0u, 0u);
     while (cur.valid()) {
       const uint32_t idc = idn;
       TileCursor nc = cur;
       nc.next(a, S, h);
-      idn = load_ids(nc);
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
@@ -444,6 +430,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       uint8_t* dst = sm + OFF_K + 2 * st * HBLK;
       const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
       const uint8_t* tab = cur.U.hb ? cur.U.hb + L.ktab : nullptr;
+      if (rank == 0 && cur.tl == 0 && cur.U.psac) {
+        // U_r^T of this chunk (rows j < r, zero up to 32) as f16 into the
+        // chunk-parity buffer read by the Q U_r MMA; published with this tile.
+        uint8_t* sU = sm + OFF_U + (cur.u & 1) * 2 * UBLK;
+        const uint8_t* ut = cur.U.hb + L.ut;
+#pragma unroll 1
+        for (int idx = kt; idx < 32 * 16; idx += 128) {
+          const int j = idx >> 4, ch = idx & 15;
+          const uint4 v = j < r ? bf16x8_to_f16x8(ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2)) : make_uint4(0u, 0u, 0u, 0u);
+          st_chunk(sU, j, ch, v, 32);
+        }
+      }
       const bool psac_lane = cur.U.psac && q * 8 < r;
       // One row per pass (loads, then its reconstruction); the pass loop is
       // kept rolled so that the four roles' hot loops stay small enough for
@@ -529,6 +527,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       }
       fence_proxy_async_smem();
       arrive_leader(B_KFULL + st);
+      // the next tile's ids and zero-points are fetched only now: a release
+      // waits for every memory operation the thread has in flight
+      idn = load_ids(nc);
       cur = nc;
       ++jt;
     }
@@ -565,7 +566,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const uint64_t idc = idn;
       TileCursor nc = cur;
       nc.next(a, S, h);
-      idn = load_ids(nc);
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
@@ -624,6 +624,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       }
       fence_proxy_async_smem();
       arrive_leader(B_VFULL + st);
+      // the next tile's ids and zero-points are fetched only now: a release
+      // waits for every memory operation the thread has in flight
+      idn = load_ids(nc);
       cur = nc;
       ++jt;
     }
@@ -637,7 +640,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     if (rank == 0 && lane == 0) {
       const uint32_t aQ = smem_u32(sm + OFF_Q), aQU = smem_u32(sm + OFF_QU);
       const uint32_t aK = smem_u32(sm + OFF_K), aC = smem_u32(sm + OFF_C), aV = smem_u32(sm + OFF_V);
+      const uint32_t aU = smem_u32(sm + OFF_U);
       constexpr uint32_t idS = idesc_f16(256, 128, false);
+      constexpr uint32_t idQU = idesc_f16(256, 64, false);
       constexpr uint32_t idPV = idesc_f16(256, 128, true);
       int total = 0;
       for (int u = 0; u < n_units; ++u) total += (unit_at(a, S, u, h).ntok + 127) / 128;
@@ -648,11 +653,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       auto issue_S = [&](int i) -> bool {
         const int st = sjt & 1;
         const uint32_t ph = (sjt >> 1) & 1;
-        if (sc.tl == 0 && (sc.u == 0 || sc.U.psac)) {
+        if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph)) return false;
+        if (sc.tl == 0 && sc.u == 0) {  // Q_i in place
           if (!mbar_wait_cluster(bar(B_QU + i), qph[i])) return false;
           qph[i] ^= 1;
         }
-        if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph)) return false;
+        if (sc.tl == 0 && sc.U.psac) {
+          // Q_i U_r of this chunk into columns 64.. of S_i (N = 64: the
+          // leader's 32 rows of U_r^T, the follower's zero rows): every MMA
+          // that read S_i or Q_i U_r of the previous chunk was issued before.
+          tc_fence_after();
+          const uint32_t aUc = aU + (sc.u & 1) * 2 * UBLK;
+#pragma unroll
+          for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+              umma2_ss(tbase + 128 * i + 64, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
+                       desc_sw128(aUc + kb * UBLK + ks * 32), idQU, (kb | ks) != 0);
+          umma2_commit_both(bar(B_QUMMA + i));
+          if (!mbar_wait_cluster(bar(B_QU + i), qph[i])) return false;  // moved into the shared A operand
+          qph[i] ^= 1;
+        }
         tc_fence_after();
         const uint32_t tS = tbase + 128 * i;
 #pragma unroll
