@@ -204,17 +204,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   // writes (the caller fences them for their consumer first).
   auto arrive_leader = [&](int i) {
     __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(mapa(bar(i), 0));
+    if (lane == 0) {
+      if (rank == 0) mbar_arrive(bar(i));
+      else mbar_arrive_cluster(mapa(bar(i), 0));
+    }
+  };
+  // Hand-off of a finished stage (KV tile or P_i) to the leader's MMA thread.
+  // In the leader each warp arrives on its own barrier b (a CTA-scope
+  // release).  In the follower the role's four warps meet at named barrier
+  // nb, which also ANDs their `ok` flags so that a timed-out wait ends the
+  // role in all four warps together, and one lane arrives for all of them
+  // with a cluster-scope release (which stalls its warp for hundreds of
+  // cycles, so the other three do not pay it).  Returns the common flag.
+  auto handoff = [&](int b, int nb, bool okw) -> bool {
+    if (rank == 0) {
+      __syncwarp();
+      if (okw && lane == 0) mbar_arrive(bar(b));
+      return okw;
+    }
+    const bool all = named_bar_and(nb, 128, okw);
+    if (all && (warp & 3) == 0 && lane == 0) mbar_arrive_cluster(mapa(bar(b), 0));
+    return all;
   };
 
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
-      mbar_init(bar(B_KFULL + s), 8);    // 4 rebuild warps x 2 CTAs (leader's copy)
+      mbar_init(bar(B_KFULL + s), 5);    // 4 leader rebuild warps + 1 follower arrival
       mbar_init(bar(B_KEMPTY + s), 1);   // pair MMA commit, both CTAs
-      mbar_init(bar(B_VFULL + s), 8);
+      mbar_init(bar(B_VFULL + s), 5);
       mbar_init(bar(B_VEMPTY + s), 1);
       mbar_init(bar(B_SFULL + s), 1);
-      mbar_init(bar(B_PFULL + s), 8);    // 4 softmax warps x 2 CTAs (leader's copy)
+      mbar_init(bar(B_PFULL + s), 5);    // 4 leader softmax warps + 1 follower arrival
       mbar_init(bar(B_QU + s), 8);
     }
     mbar_init(bar(B_OFINAL), 1);
@@ -251,14 +271,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     // moves it into the shared A operand of the extra reduction columns.
     uint32_t qum = 0;  // completed Q_i U_r MMAs
     auto take_qu = [&]() -> bool {
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1))) return false;
-      ++qum;
-      tc_fence_after();
-      qu_to_smem(sm + OFF_QU, i, row, tS + 64, rpad);
-      tc_fence_before();
-      fence_proxy_async_smem();
-      arrive_leader(B_QU + i);
-      return true;
+      bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1));
+      if (okw) {
+        ++qum;
+        tc_fence_after();
+        qu_to_smem(sm + OFF_QU, i, row, tS + 64, rpad);
+        tc_fence_before();
+        fence_proxy_async_smem();
+      }
+      if (rank == 1) okw = named_bar_and(1 + i, 128, okw);  // the group leaves together
+      if (okw) arrive_leader(B_QU + i);
+      return okw;
     };
 
     const float sl2 = a.sm_scale * 1.4426950408889634f;
@@ -271,92 +294,94 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int ntiles = (U.ntok + 127) / 128;
       for (int tl = 0; tl < ntiles; ++tl, ++jt) {
         const int nvalid = min(128, U.ntok - tl * 128);
-        ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1));
-        if (!ok) break;
-        tc_fence_after();
-        // ---- row maximum: the four 32-column blocks of S_i, two loads per wait
-        float va[32], vb[32];
-        float mt = -INFINITY;
-        if (nvalid == 128) {  // the TMEM loads reduce the columns they read
-          float m0, m1, m2, m3;
-          tmem_max32x2(tS, tS + 32, m0, m1);
-          tmem_max32x2(tS + 64, tS + 96, m2, m3);
-          mt = fmax3(fmaxf(m0, m1), m2, m3);
-        } else {
-#pragma unroll 1
+        const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1));
+        if (okw) {
+          tc_fence_after();
+          // ---- row maximum: the four 32-column blocks of S_i, two loads per wait
+          float va[32], vb[32];
+          float mt = -INFINITY;
+          if (nvalid == 128) {  // the TMEM loads reduce the columns they read
+            float m0, m1, m2, m3;
+            tmem_max32x2(tS, tS + 32, m0, m1);
+            tmem_max32x2(tS + 64, tS + 96, m2, m3);
+            mt = fmax3(fmaxf(m0, m1), m2, m3);
+          } else {
+  #pragma unroll 1
+            for (int cp = 0; cp < 2; ++cp) {
+              tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
+  #pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                if (64 * cp + e < nvalid) mt = fmaxf(mt, va[e]);
+                if (64 * cp + 32 + e < nvalid) mt = fmaxf(mt, vb[e]);
+              }
+            }
+          }
+          const float m_new = fmaxf(m_run, mt);
+          const bool need = (m_new - m_run) * sl2 > kTauLog2;
+          float alpha = 1.0f;
+          if (need) {
+            alpha = ex2((m_run - m_new) * sl2);
+            m_run = m_new;
+            l_run *= alpha;
+          }
+          // S_i of this tile completing implies the previous P_i V MMA is done,
+          // so O_i can be rescaled here.
+          if (__any_sync(0xFFFFFFFFu, need) && jt > 0) {
+  #pragma unroll 1
+            for (int cb = 0; cb < 4; ++cb) {
+              tmem_ld32(tO + cb * 32, va);
+  #pragma unroll
+              for (int e = 0; e < 32; ++e) va[e] *= alpha;
+              tmem_st32(tO + cb * 32, va);
+            }
+          }
+          // ---- P = exp2(s * scale * log2(e) - m) as f16 pairs (one MUFU op per
+          // pair), written over the S columns already read; the row sum adds
+          // exactly those f16 values, 32 at a time in a packed f16 tree (each
+          // partial <= 32 * 2^8, exact to 2^-11 relative), then in fp32.
+          const float mb = m_run * sl2;
+          const uint64_t SL = splat2(sl2), MB = splat2(-mb);
+          float lsum = 0.0f;
+          auto exp_block = [&](const float (&v)[32], uint32_t (&pk)[16], int col0, bool full) {
+  #pragma unroll
+            for (int e = 0; e < 32; e += 2) {
+              float x0 = v[e], x1 = v[e + 1];
+              fma2(x0, x1, SL, MB);
+              if (!full) {
+                if (col0 + e >= nvalid) x0 = -INFINITY;
+                if (col0 + e + 1 >= nvalid) x1 = -INFINITY;
+              }
+              pk[e >> 1] = ex2_f16x2(pack_f16(x0, x1));
+            }
+          };
+          auto sum_block = [&](const uint32_t (&pk)[16]) -> float {
+            __half2 t8[8];
+  #pragma unroll
+            for (int k = 0; k < 8; ++k) t8[k] = __hadd2(u2h(pk[2 * k]), u2h(pk[2 * k + 1]));
+  #pragma unroll
+            for (int k = 0; k < 4; ++k) t8[k] = __hadd2(t8[2 * k], t8[2 * k + 1]);
+            t8[0] = __hadd2(t8[0], t8[1]);
+            t8[2] = __hadd2(t8[2], t8[3]);
+            const float2 f = __half22float2(__hadd2(t8[0], t8[2]));
+            return f.x + f.y;
+          };
+  #pragma unroll 1
           for (int cp = 0; cp < 2; ++cp) {
             tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              if (64 * cp + e < nvalid) mt = fmaxf(mt, va[e]);
-              if (64 * cp + 32 + e < nvalid) mt = fmaxf(mt, vb[e]);
-            }
+            uint32_t pk[16];
+            exp_block(va, pk, 64 * cp, nvalid == 128);
+            tmem_st16(tS + 32 * cp, pk);  // P of columns 64cp..64cp+31 over columns already read
+            lsum += sum_block(pk);
+            exp_block(vb, pk, 64 * cp + 32, nvalid == 128);
+            tmem_st16(tS + 32 * cp + 16, pk);
+            lsum += sum_block(pk);
           }
+          tmem_wait_st();
+          l_run += lsum;
+          tc_fence_before();
         }
-        const float m_new = fmaxf(m_run, mt);
-        const bool need = (m_new - m_run) * sl2 > kTauLog2;
-        float alpha = 1.0f;
-        if (need) {
-          alpha = ex2((m_run - m_new) * sl2);
-          m_run = m_new;
-          l_run *= alpha;
-        }
-        // S_i of this tile completing implies the previous P_i V MMA is done,
-        // so O_i can be rescaled here.
-        if (__any_sync(0xFFFFFFFFu, need) && jt > 0) {
-#pragma unroll 1
-          for (int cb = 0; cb < 4; ++cb) {
-            tmem_ld32(tO + cb * 32, va);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) va[e] *= alpha;
-            tmem_st32(tO + cb * 32, va);
-          }
-        }
-        // ---- P = exp2(s * scale * log2(e) - m) as f16 pairs (one MUFU op per
-        // pair), written over the S columns already read; the row sum adds
-        // exactly those f16 values, 32 at a time in a packed f16 tree (each
-        // partial <= 32 * 2^8, exact to 2^-11 relative), then in fp32.
-        const float mb = m_run * sl2;
-        const uint64_t SL = splat2(sl2), MB = splat2(-mb);
-        float lsum = 0.0f;
-        auto exp_block = [&](const float (&v)[32], uint32_t (&pk)[16], int col0, bool full) {
-#pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            float x0 = v[e], x1 = v[e + 1];
-            fma2(x0, x1, SL, MB);
-            if (!full) {
-              if (col0 + e >= nvalid) x0 = -INFINITY;
-              if (col0 + e + 1 >= nvalid) x1 = -INFINITY;
-            }
-            pk[e >> 1] = ex2_f16x2(pack_f16(x0, x1));
-          }
-        };
-        auto sum_block = [&](const uint32_t (&pk)[16]) -> float {
-          __half2 t8[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) t8[k] = __hadd2(u2h(pk[2 * k]), u2h(pk[2 * k + 1]));
-#pragma unroll
-          for (int k = 0; k < 4; ++k) t8[k] = __hadd2(t8[2 * k], t8[2 * k + 1]);
-          t8[0] = __hadd2(t8[0], t8[1]);
-          t8[2] = __hadd2(t8[2], t8[3]);
-          const float2 f = __half22float2(__hadd2(t8[0], t8[2]));
-          return f.x + f.y;
-        };
-#pragma unroll 1
-        for (int cp = 0; cp < 2; ++cp) {
-          tmem_ld32x2(tS + 64 * cp, tS + 64 * cp + 32, va, vb);
-          uint32_t pk[16];
-          exp_block(va, pk, 64 * cp, nvalid == 128);
-          tmem_st16(tS + 32 * cp, pk);  // P of columns 64cp..64cp+31 over columns already read
-          lsum += sum_block(pk);
-          exp_block(vb, pk, 64 * cp + 32, nvalid == 128);
-          tmem_st16(tS + 32 * cp + 16, pk);
-          lsum += sum_block(pk);
-        }
-        tmem_wait_st();
-        l_run += lsum;
-        tc_fence_before();
-        arrive_leader(B_PFULL + i);
+        ok = handoff(B_PFULL + i, 1 + i, okw);
+        if (!ok) break;
       }
       if (ok && u + 1 < n_units && unit_at(a, S, u + 1, h).psac) ok = take_qu();
     }
@@ -423,110 +448,109 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
-      if (!mbar_wait(bar(B_KEMPTY + st), ph ^ 1)) {
-        ok = false;
-        break;
-      }
-      uint8_t* dst = sm + OFF_K + 2 * st * HBLK;
-      const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
-      const uint8_t* tab = cur.U.hb ? cur.U.hb + L.ktab : nullptr;
-      if (rank == 0 && cur.tl == 0 && cur.U.psac) {
-        // U_r^T of this chunk (rows j < r, zero up to 32) as f16 into the
-        // chunk-parity buffer read by the Q U_r MMA; published with this tile.
-        uint8_t* sU = sm + OFF_U + (cur.u & 1) * 2 * UBLK;
-        const uint8_t* ut = cur.U.hb + L.ut;
-#pragma unroll 1
-        for (int idx = kt; idx < 32 * 16; idx += 128) {
-          const int j = idx >> 4, ch = idx & 15;
-          const uint4 v = j < r ? bf16x8_to_f16x8(ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2)) : make_uint4(0u, 0u, 0u, 0u);
-          st_chunk(sU, j, ch, v, 32);
+      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_KEMPTY + st), ph ^ 1));
+      if (okw) {
+        uint8_t* dst = sm + OFF_K + 2 * st * HBLK;
+        const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
+        const uint8_t* tab = cur.U.hb ? cur.U.hb + L.ktab : nullptr;
+        if (rank == 0 && cur.tl == 0 && cur.U.psac) {
+          // U_r^T of this chunk (rows j < r, zero up to 32) as f16 into the
+          // chunk-parity buffer read by the Q U_r MMA; published with this tile.
+          uint8_t* sU = sm + OFF_U + (cur.u & 1) * 2 * UBLK;
+          const uint8_t* ut = cur.U.hb + L.ut;
+  #pragma unroll 1
+          for (int idx = kt; idx < 32 * 16; idx += 128) {
+            const int j = idx >> 4, ch = idx & 15;
+            const uint4 v = j < r ? bf16x8_to_f16x8(ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2)) : make_uint4(0u, 0u, 0u, 0u);
+            st_chunk(sU, j, ch, v, 32);
+          }
         }
-      }
-      const bool psac_lane = cur.U.psac && q * 8 < r;
-      // One row per pass (loads, then its reconstruction); the pass loop is
-      // kept rolled so that the four roles' hot loops stay small enough for
-      // the instruction caches.
-#pragma unroll 1
-      for (int p = 0; p < 2; ++p) {
-        const int lr = wrow + 8 * p, trw = tro + lr;
-        const bool rv = trw < nv;
-        uint32_t mv[2][8];  // [slice][words]
-        uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
-        uint2 cfv = make_uint2(0u, 0u);  // PSAC INT8 codes 8q..8q+7 of the row
-        uint32_t sgv = 0u;               // PSAC row scale (binary16 bits)
-#pragma unroll
-        for (int sl = 0; sl < 2; ++sl)
-#pragma unroll
-          for (int e = 0; e < 8; ++e) mv[sl][e] = 0u;
-        if (rv) {
-          if (tb) {
-            const uint8_t* mu = tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256;
-            ldg32B(mu + 32 * q, mv[0]);
-            ldg32B(mu + 128 + 32 * q, mv[1]);
-            const uint8_t* cp = tb + L.k_codes + trw * 32;
-            cwv[0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
-            cwv[1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
-            const unsigned short* sp = reinterpret_cast<const unsigned short*>(tb + L.k_scales + (int64_t)trw * L.ng * 2);
-            scv[0] = __ldg(sp + ((16 * q) >> gshift));
-            scv[1] = __ldg(sp + ((64 + 16 * q) >> gshift));
-            if (psac_lane) {
-              cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
-              sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
+        const bool psac_lane = cur.U.psac && q * 8 < r;
+        // One row per pass (loads, then its reconstruction); the pass loop is
+        // kept rolled so that the four roles' hot loops stay small enough for
+        // the instruction caches.
+  #pragma unroll 1
+        for (int p = 0; p < 2; ++p) {
+          const int lr = wrow + 8 * p, trw = tro + lr;
+          const bool rv = trw < nv;
+          uint32_t mv[2][8];  // [slice][words]
+          uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
+          uint2 cfv = make_uint2(0u, 0u);  // PSAC INT8 codes 8q..8q+7 of the row
+          uint32_t sgv = 0u;               // PSAC row scale (binary16 bits)
+  #pragma unroll
+          for (int sl = 0; sl < 2; ++sl)
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) mv[sl][e] = 0u;
+          if (rv) {
+            if (tb) {
+              const uint8_t* mu = tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256;
+              ldg32B(mu + 32 * q, mv[0]);
+              ldg32B(mu + 128 + 32 * q, mv[1]);
+              const uint8_t* cp = tb + L.k_codes + trw * 32;
+              cwv[0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
+              cwv[1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
+              const unsigned short* sp = reinterpret_cast<const unsigned short*>(tb + L.k_scales + (int64_t)trw * L.ng * 2);
+              scv[0] = __ldg(sp + ((16 * q) >> gshift));
+              scv[1] = __ldg(sp + ((64 + 16 * q) >> gshift));
+              if (psac_lane) {
+                cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
+                sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
+              }
+            } else {
+              const __nv_bfloat16* src = a.kcur + ((size_t)(cur.tl * 128 + trw) * H + h) * 128;
+  #pragma unroll
+              for (int sl = 0; sl < 2; ++sl) {
+                const uint4 f0 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q));
+                const uint4 f1 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q + 8));
+                mv[sl][0] = f0.x; mv[sl][1] = f0.y; mv[sl][2] = f0.z; mv[sl][3] = f0.w;
+                mv[sl][4] = f1.x; mv[sl][5] = f1.y; mv[sl][6] = f1.z; mv[sl][7] = f1.w;
+              }
             }
-          } else {
-            const __nv_bfloat16* src = a.kcur + ((size_t)(cur.tl * 128 + trw) * H + h) * 128;
-#pragma unroll
-            for (int sl = 0; sl < 2; ++sl) {
-              const uint4 f0 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q));
-              const uint4 f1 = bf16x8_to_f16x8(ldg16(src + 64 * sl + 16 * q + 8));
-              mv[sl][0] = f0.x; mv[sl][1] = f0.y; mv[sl][2] = f0.z; mv[sl][3] = f0.w;
-              mv[sl][4] = f1.x; mv[sl][5] = f1.y; mv[sl][6] = f1.z; mv[sl][7] = f1.w;
+          }
+          const bool deq = tb && rv;
+          const uint32_t zbyte = (idc >> (16 + 8 * p)) & 0xFFu;
+  #pragma unroll
+          for (int sl = 0; sl < 2; ++sl) {
+            const int c0 = 8 * sl + 2 * q;  // first of the two chunks of this slice
+            // f16 pairs mu + (q - z) s; a row of the active chunk (or a padding
+            // row) passes through with s = 0 and z = q.
+            const int g = (64 * sl + 16 * q) >> gshift;
+            const uint32_t sb = deq ? scv[sl] : 0u;
+            const __half2 s2 = u2h(sb | (sb << 16));
+            const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
+            const __half2 z2 = u2h(zz | (zz << 16));
+            const uint32_t word = cwv[sl];
+            uint32_t ow[8];
+  #pragma unroll
+            for (int k = 0; k < 8; ++k) {  // channel pairs (2k, 2k+1) of the 16-channel word
+              const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+              ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[sl][k])));
             }
+            st_chunk(dst, lr, c0, make_uint4(ow[0], ow[1], ow[2], ow[3]), 64);
+            st_chunk(dst, lr, c0 + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]), 64);
+          }
+          if (cur.U.psac && q * 8 < rpad) {
+            // C_hat = t * sigma (Eq. 16), PSAC columns 8q..8q+7 of the row, in
+            // f16: byte b of an INT8 code t becomes the f16 1024 + (t + 128)
+            // (its byte XOR 0x80 under exponent bits 0x64), minus 1152 gives t
+            // exactly, and one f16 multiply rounds t * sigma once.  Lanes past
+            // r and padding rows hold zero codes and scale: zero columns.
+            const __half2 sg2 = u2h(sgv | (sgv << 16));
+            const __half2 off2 = u2h(0x64806480u);  // (1152, 1152)
+            const uint32_t cwd[2] = {cfv.x ^ 0x80808080u, cfv.y ^ 0x80808080u};
+            uint32_t w4[4];
+  #pragma unroll
+            for (int q2 = 0; q2 < 4; ++q2) {
+              const uint32_t b0 = 2 * (q2 & 1);
+              const uint32_t t2 = __byte_perm(cwd[q2 >> 1], 0x64646464u, b0 | (4u << 4) | ((b0 + 1) << 8) | (4u << 12));
+              w4[q2] = h2u(__hmul2(__hsub2(u2h(t2), off2), sg2));
+            }
+            st_chunk(sm + OFF_C, lr, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]), 64);
           }
         }
-        const bool deq = tb && rv;
-        const uint32_t zbyte = (idc >> (16 + 8 * p)) & 0xFFu;
-#pragma unroll
-        for (int sl = 0; sl < 2; ++sl) {
-          const int c0 = 8 * sl + 2 * q;  // first of the two chunks of this slice
-          // f16 pairs mu + (q - z) s; a row of the active chunk (or a padding
-          // row) passes through with s = 0 and z = q.
-          const int g = (64 * sl + 16 * q) >> gshift;
-          const uint32_t sb = deq ? scv[sl] : 0u;
-          const __half2 s2 = u2h(sb | (sb << 16));
-          const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
-          const __half2 z2 = u2h(zz | (zz << 16));
-          const uint32_t word = cwv[sl];
-          uint32_t ow[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {  // channel pairs (2k, 2k+1) of the 16-channel word
-            const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
-            ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[sl][k])));
-          }
-          st_chunk(dst, lr, c0, make_uint4(ow[0], ow[1], ow[2], ow[3]), 64);
-          st_chunk(dst, lr, c0 + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]), 64);
-        }
-        if (cur.U.psac && q * 8 < rpad) {
-          // C_hat = t * sigma (Eq. 16), PSAC columns 8q..8q+7 of the row, in
-          // f16: byte b of an INT8 code t becomes the f16 1024 + (t + 128)
-          // (its byte XOR 0x80 under exponent bits 0x64), minus 1152 gives t
-          // exactly, and one f16 multiply rounds t * sigma once.  Lanes past
-          // r and padding rows hold zero codes and scale: zero columns.
-          const __half2 sg2 = u2h(sgv | (sgv << 16));
-          const __half2 off2 = u2h(0x64806480u);  // (1152, 1152)
-          const uint32_t cwd[2] = {cfv.x ^ 0x80808080u, cfv.y ^ 0x80808080u};
-          uint32_t w4[4];
-#pragma unroll
-          for (int q2 = 0; q2 < 4; ++q2) {
-            const uint32_t b0 = 2 * (q2 & 1);
-            const uint32_t t2 = __byte_perm(cwd[q2 >> 1], 0x64646464u, b0 | (4u << 4) | ((b0 + 1) << 8) | (4u << 12));
-            w4[q2] = h2u(__hmul2(__hsub2(u2h(t2), off2), sg2));
-          }
-          st_chunk(sm + OFF_C, lr, (st * rpad) / 8 + q, make_uint4(w4[0], w4[1], w4[2], w4[3]), 64);
-        }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
-      arrive_leader(B_KFULL + st);
+      if (!(ok = handoff(B_KFULL + st, 3, okw))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
@@ -569,61 +593,60 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
-      if (!mbar_wait(bar(B_VEMPTY + st), ph ^ 1)) {
-        ok = false;
-        break;
-      }
-      uint8_t* dst = sm + OFF_V + st * BLK;
-      const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
-      const uint8_t* tab = cur.U.hb ? cur.U.hb + L.vtab : nullptr;
-      const int g = (16 * c16) >> gshift;
-#pragma unroll 1
-      for (int rd = 0; rd < 2; ++rd) {
-        uint32_t mv[2][8];
-        uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
-#pragma unroll
-        for (int pp = 0; pp < 2; ++pp) {
-          const int p = 2 * rd + pp;
-          const int row = wrow + 8 * p;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) mv[pp][e] = 0u;
-          if (row < nv) {
-            if (tb) {
-              ldg32B(tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256 + 32 * c16, mv[pp]);
-              cwv[pp] = __ldg(reinterpret_cast<const uint32_t*>(tb + L.v_codes + row * 32 + 4 * c16));
-              scv[pp] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.v_scales + (int64_t)row * L.ng * 2) + g);
-            } else {
-              const __nv_bfloat16* src = a.vcur + ((size_t)(cur.tl * 128 + row) * H + h) * 128 + 16 * c16;
-              const uint4 f0 = bf16x8_to_f16x8(ldg16(src)), f1 = bf16x8_to_f16x8(ldg16(src + 8));
-              mv[pp][0] = f0.x; mv[pp][1] = f0.y; mv[pp][2] = f0.z; mv[pp][3] = f0.w;
-              mv[pp][4] = f1.x; mv[pp][5] = f1.y; mv[pp][6] = f1.z; mv[pp][7] = f1.w;
+      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_VEMPTY + st), ph ^ 1));
+      if (okw) {
+        uint8_t* dst = sm + OFF_V + st * BLK;
+        const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
+        const uint8_t* tab = cur.U.hb ? cur.U.hb + L.vtab : nullptr;
+        const int g = (16 * c16) >> gshift;
+  #pragma unroll 1
+        for (int rd = 0; rd < 2; ++rd) {
+          uint32_t mv[2][8];
+          uint32_t cwv[2] = {0u, 0u}, scv[2] = {0u, 0u};
+  #pragma unroll
+          for (int pp = 0; pp < 2; ++pp) {
+            const int p = 2 * rd + pp;
+            const int row = wrow + 8 * p;
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) mv[pp][e] = 0u;
+            if (row < nv) {
+              if (tb) {
+                ldg32B(tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256 + 32 * c16, mv[pp]);
+                cwv[pp] = __ldg(reinterpret_cast<const uint32_t*>(tb + L.v_codes + row * 32 + 4 * c16));
+                scv[pp] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.v_scales + (int64_t)row * L.ng * 2) + g);
+              } else {
+                const __nv_bfloat16* src = a.vcur + ((size_t)(cur.tl * 128 + row) * H + h) * 128 + 16 * c16;
+                const uint4 f0 = bf16x8_to_f16x8(ldg16(src)), f1 = bf16x8_to_f16x8(ldg16(src + 8));
+                mv[pp][0] = f0.x; mv[pp][1] = f0.y; mv[pp][2] = f0.z; mv[pp][3] = f0.w;
+                mv[pp][4] = f1.x; mv[pp][5] = f1.y; mv[pp][6] = f1.z; mv[pp][7] = f1.w;
+              }
             }
           }
-        }
-#pragma unroll
-        for (int pp = 0; pp < 2; ++pp) {
-          const int p = 2 * rd + pp;
-          const int row = wrow + 8 * p;
-          // mu + (q - z) s; active-chunk and padding rows pass through with
-          // s = 0 and zero codes and zero-points (the ids word is 0 there).
-          const uint32_t zbyte = (uint32_t)((idc >> (32 + 8 * p)) & 0xFFu);
-          const uint32_t sb = scv[pp];
-          const __half2 s2 = u2h(sb | (sb << 16));
-          const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
-          const __half2 z2 = u2h(zz | (zz << 16));
-          const uint32_t word = cwv[pp];
-          uint32_t ow[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
-            ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[pp][k])));
+  #pragma unroll
+          for (int pp = 0; pp < 2; ++pp) {
+            const int p = 2 * rd + pp;
+            const int row = wrow + 8 * p;
+            // mu + (q - z) s; active-chunk and padding rows pass through with
+            // s = 0 and zero codes and zero-points (the ids word is 0 there).
+            const uint32_t zbyte = (uint32_t)((idc >> (32 + 8 * p)) & 0xFFu);
+            const uint32_t sb = scv[pp];
+            const __half2 s2 = u2h(sb | (sb << 16));
+            const uint32_t zz = 0x6400u | ((zbyte >> (2 * g)) & 3u);
+            const __half2 z2 = u2h(zz | (zz << 16));
+            const uint32_t word = cwv[pp];
+            uint32_t ow[8];
+  #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t qq = ((word >> (2 * k)) & 0x00030003u) | 0x64006400u;
+              ow[k] = h2u(__hfma2(__hsub2(u2h(qq), z2), s2, u2h(mv[pp][k])));
+            }
+            st_chunk(dst, row, 2 * q, make_uint4(ow[0], ow[1], ow[2], ow[3]));
+            st_chunk(dst, row, 2 * q + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]));
           }
-          st_chunk(dst, row, 2 * q, make_uint4(ow[0], ow[1], ow[2], ow[3]));
-          st_chunk(dst, row, 2 * q + 1, make_uint4(ow[4], ow[5], ow[6], ow[7]));
         }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
-      arrive_leader(B_VFULL + st);
+      if (!(ok = handoff(B_VFULL + st, 4, okw))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
