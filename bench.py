@@ -350,7 +350,7 @@ def oracle_sample(wl, append_tokens, attend_rows, attend_heads, nthreads):
     return full, desc, (t_app + t_att)
 
 
-def cpu_baseline(wl, nthreads, append_tokens=512, attend_rows=32, attend_heads=4):
+def cpu_baseline(wl, nthreads, append_tokens=4680, attend_rows=2048, attend_heads=8):
     from oracle import oracle as orc
     cores = nthreads if nthreads > 0 else orc.max_threads()
     full, desc, spent = oracle_sample(wl, append_tokens, attend_rows, attend_heads, nthreads)
@@ -393,11 +393,16 @@ def main():
     ap.add_argument("--workload", default="wan14b_layer")
     ap.add_argument("--cpu-threads", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--heads", type=int, default=0,
+                    help="profiling only: the workload with fewer heads (same per-head work); not a bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from paper_2609_26425_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
+    if args.heads > 0:
+        import dataclasses
+        wl = dataclasses.replace(wl, heads=args.heads, name=f"{wl.name}_h{args.heads}")
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
 
