@@ -188,12 +188,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const Layout& L = a.L;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // Grid: x = 2 * (block of 512 queries) + rank (the CTA pair of a cluster),
+  // y = head (the pairs of one head run close together and share its packed
+  // tiles through L2).
   const int h = blockIdx.y;
   const int H = L.H, r = L.r;
   const int rpad = r == 8 ? 16 : r;
   const int gshift = L.G == 32 ? 5 : 6;
   const uint32_t rank = cluster_rank();  // 0: leader
-  const int64_t q0 = (int64_t)blockIdx.x * 256;
+  const int64_t pair0 = (int64_t)(blockIdx.x >> 1) * 512;
+  const int64_t q0 = pair0 + 256 * rank;
+  // Q tiles the pair runs: the second is left out when neither CTA has a
+  // query in it (the tail of the query range), halving that pair's MMA and
+  // softmax work.
+  const int nqt = pair0 + 128 < a.Nq ? 2 : 1;
   const int n_units = S.n + (a.Ncur > 0 ? 1 : 0);
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
@@ -269,6 +277,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     // Q_i U_r of each chunk that carries PSAC columns: the MMA thread computes
     // it into columns 64.. of S_i (free while S_i is not in use); this group
     // moves it into the shared A operand of the extra reduction columns.
+    if (i < nqt) {
     uint32_t qum = 0;  // completed Q_i U_r MMAs
     auto take_qu = [&]() -> bool {
       bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1));
@@ -406,6 +415,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       if (a.lse && qvalid) a.lse[(size_t)h * a.Nq + qi] = m_run * a.sm_scale + logf(l_run);
     } else {
       *s_err = 1;
+    }
     }
   } else if (warp < W_DQV) {
     // ------------------------------------------------------------ K_hat0 + C_hat of this CTA's 64 keys (warps 8-11)
@@ -709,27 +719,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           for (int ks = 0; ks < rpad / 16; ++ks)
             umma2_ss(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32), idS, 1u);
         umma2_commit_both(bar(B_SFULL + i));
-        if (i == 1) {
+        if (i == nqt - 1) {
           umma2_commit_both(bar(B_KEMPTY + st));
           sc.next(a, S, h);
           ++sjt;
         }
         return true;
       };
-      if (total > 0) ok = issue_S(0) && issue_S(1);
+      if (total > 0) ok = issue_S(0) && (nqt == 1 || issue_S(1));
       for (int jt = 0; jt < total && ok; ++jt) {
         const int st = jt & 1;
         const uint32_t ph = (jt >> 1) & 1;
         if (!(ok = mbar_wait_cluster(bar(B_VFULL + st), ph))) break;
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < nqt; ++i) {
           if (!(ok = mbar_wait_cluster(bar(B_PFULL + i), jt & 1))) break;
           tc_fence_after();
           const uint32_t tP = tbase + 128 * i, tO = tbase + 256 + 128 * i;
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks)
             umma2_ts(tO, tP + 8 * ks, desc_sw128(aV + st * BLK + ks * 2048), idPV, (jt > 0 || ks > 0) ? 1u : 0u);
-          if (i == 1) umma2_commit_both(bar(B_VEMPTY + st));
+          if (i == nqt - 1) umma2_commit_both(bar(B_VEMPTY + st));
           if (jt + 1 < total && !(ok = issue_S(i))) break;
         }
       }
