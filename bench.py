@@ -141,6 +141,23 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# ---------------------------------------------------------------------------- replicas
+def job_time_ms(local_ms, world, device):
+    """The whole job's time: the slowest rank's (max over ranks; one rank: its own)."""
+    if world <= 1:
+        return float(local_ms)
+    import torch
+    tt = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+    return float(tt.item())
+
+
+def whole_job_tflops(world, steps, flops_per_step, job_ms):
+    """Whole-job throughput of `world` replicas, each doing `steps` steps of
+    `flops_per_step` (weak scaling), over the slowest rank's time."""
+    return world * steps * flops_per_step / (job_ms * 1e-3) / 1e12
+
+
 # ---------------------------------------------------------------------------- GPU arm
 def run_gpu(args, wl, rank, world):
     import torch
@@ -223,10 +240,7 @@ def run_gpu(args, wl, rank, world):
     ms = t0.elapsed_time(t1)
     att_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
     app_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = job_time_ms(ms, world, dev)
 
     # ---- end to end through the public API with host buffers
     pin = lambda t: t.pin_memory()
@@ -264,16 +278,13 @@ def run_gpu(args, wl, rank, world):
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([e_ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        e_ms = float(tt.item())
+    e_ms = job_time_ms(e_ms, world, dev)
 
     pk = peaks()
     att_tflops = nums["attend_flops"] / (att_ms * 1e-3) / 1e12
     app_gbs = nums["append_bytes"] / (app_ms * 1e-3) / 1e9
-    value = world * args.steps * nums["attend_flops"] / (ms * 1e-3) / 1e12
-    e2e_value = world * args.steps * nums["attend_flops"] / (e_ms * 1e-3) / 1e12
+    value = whole_job_tflops(world, args.steps, nums["attend_flops"], ms)
+    e2e_value = whole_job_tflops(world, args.steps, nums["attend_flops"], e_ms)
     res = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
