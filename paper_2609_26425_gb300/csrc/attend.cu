@@ -306,14 +306,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1));
         if (okw) {
           tc_fence_after();
-          // ---- row maximum: the four 32-column blocks of S_i, two loads per wait
+          // ---- row maximum: four reducing TMEM loads and one wait
+          const bool full = nvalid == 128;
           float va[32], vb[32];
           float mt = -INFINITY;
-          if (nvalid == 128) {  // the TMEM loads reduce the columns they read
-            float m0, m1, m2, m3;
-            tmem_max32x2(tS, tS + 32, m0, m1);
-            tmem_max32x2(tS + 64, tS + 96, m2, m3);
-            mt = fmax3(fmaxf(m0, m1), m2, m3);
+          if (full) {
+            mt = tmem_max128(tS);
           } else {
   #pragma unroll 1
             for (int cp = 0; cp < 2; ++cp) {
@@ -337,11 +335,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           // so O_i can be rescaled here.
           if (__any_sync(0xFFFFFFFFu, need) && jt > 0) {
   #pragma unroll 1
-            for (int cb = 0; cb < 4; ++cb) {
-              tmem_ld32(tO + cb * 32, va);
+            for (int cb = 0; cb < 8; ++cb) {
+              uint32_t t[16];
+              tmem_ld16(tO + cb * 16, t);
   #pragma unroll
-              for (int e = 0; e < 32; ++e) va[e] *= alpha;
-              tmem_st32(tO + cb * 32, va);
+              for (int e = 0; e < 16; ++e) t[e] = __float_as_uint(__uint_as_float(t[e]) * alpha);
+              tmem_st16(tO + cb * 16, t);
             }
           }
           // ---- P = exp2(s * scale * log2(e) - m) as f16 pairs (one MUFU op per
