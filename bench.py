@@ -242,39 +242,62 @@ def run_gpu(args, wl, rank, world):
     app_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / args.steps
     ms = job_time_ms(ms, world, dev)
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API with host buffers: every step
+    # copies its inputs from pinned host memory and reads its output back; two
+    # device buffer sets let the copies of one step overlap the kernels of the
+    # previous one (copy-in, compute and copy-out on three streams)
     pin = lambda t: t.pin_memory()
     hq, hk, hv = pin(q), pin(k), pin(v)
     hkc, hvc = pin(kc.cpu()), pin(vc.cpu())
     hw = pin(w) if w is not None else None
     hU = pin(U) if U is not None else None
-    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
-    dkc, dvc = torch.empty_like(kc), torch.empty_like(vc)
-    dw = torch.empty_like(wd) if wd is not None else None
-    dU = torch.empty_like(Ud) if Ud is not None else None
-    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hkc, hvc) if t is not None)
-    h2d += sum(t.numel() * t.element_size() for t in (hw, hU) if t is not None)
-    d2h = hout.numel() * hout.element_size()
+    hin = (hq, hk, hv, hkc, hvc, hw, hU)
+    like = (qd, kd, vd, kc, vc, wd, Ud)
+    sets = [[torch.empty_like(t) if t is not None else None for t in like] for _ in range(2)]
+    outs = [torch.empty_like(qd) for _ in range(2)]
+    houts = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+    h2d = sum(t.numel() * t.element_size() for t in hin if t is not None)
+    d2h = houts[0].numel() * houts[0].element_size()
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]
+    ev_done = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(2)]
+    for e in ev_done + ev_out:
+        e.record(stream)
 
-    def e2e_step():
-        for h_, d_ in ((hq, dq), (hk, dk), (hv, dv), (hkc, dkc), (hvc, dvc), (hw, dw), (hU, dU)):
-            if h_ is not None:
-                d_.copy_(h_, non_blocking=True)
-        qwm.qwm_attend(cfg, hist, dq, dk, dv, out=out)
-        qwm.qwm_quantize_append(cfg, ring, dk, dv, dkc, dvc, w=dw, U=dU)
-        hout.copy_(out, non_blocking=True)
+    def e2e_step(step):
+        b = step & 1
+        dq_, dk_, dv_, dkc_, dvc_, dw_, dU_ = sets[b]
+        with torch.cuda.stream(s_in):
+            s_in.wait_event(ev_done[b])  # the kernels that read this buffer set two steps ago are done
+            for h_, d_ in zip(hin, sets[b]):
+                if h_ is not None:
+                    d_.copy_(h_, non_blocking=True)
+            ev_in[b].record(s_in)
+        stream.wait_event(ev_in[b])
+        stream.wait_event(ev_out[b])  # the output buffer's previous read-back is done
+        qwm.qwm_attend(cfg, hist, dq_, dk_, dv_, out=outs[b])
+        qwm.qwm_quantize_append(cfg, ring, dk_, dv_, dkc_, dvc_, w=dw_, U=dU_)
+        ev_done[b].record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(ev_done[b])
+            houts[b].copy_(outs[b], non_blocking=True)
+            ev_out[b].record(s_out)
 
-    for _ in range(max(1, args.warmup)):
-        e2e_step()
+    for i_ in range(max(1, args.warmup)):
+        e2e_step(i_)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        e2e_step()
+    s_in.wait_stream(stream)
+    s_out.wait_stream(stream)
+    for i_ in range(args.steps):
+        e2e_step(i_)
+    stream.wait_stream(s_in)
+    stream.wait_stream(s_out)
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = e0.elapsed_time(e1)
