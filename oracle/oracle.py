@@ -234,14 +234,22 @@ def query_stats(q_bits, r: int):
     Sec. 4.1 Eq. 8: w_hc = M_cc / ((1/d) sum_c' M_c'c');
     Sec. 4.2 Eq. 15: M_h = U Lambda U^T with eigenvalues in decreasing order,
     U_r = the first r eigenvectors (numpy.linalg.eigh as the eigen solver).
+    N = 0 (no Query yet) gives w = 1 and U = 0 (App. C.3 cold start).
     q_bits: uint16 [N][H][d].  Returns (M [H][d][d], w [H][d] fp32,
     U [H][d][r] fp64, eigenvalues [H][d] descending).
     """
     q = bf16_to_f32(q_bits).astype(np.float64)
     N, H, d = q.shape
+    if N == 0:
+        # No Query seen yet (App. C.3 cold start): uniform sensitivity and no
+        # principal subspace, so w = 1 and U = 0.
+        return (np.zeros((H, d, d)), np.ones((H, d), np.float32), np.zeros((H, d, r)), np.zeros((H, d)))
     M = np.einsum("nhc,nhe->hce", q, q) / N
     diag = np.einsum("hcc->hc", M)
-    w = (diag / diag.mean(axis=-1, keepdims=True)).astype(np.float32)
+    mean = diag.mean(axis=-1, keepdims=True)
+    # Eq. 8 is 0/0 when every past Query of a head is zero; that head falls
+    # back to the cold-start weights w = 1 (App. C.3).
+    w = np.where(mean > 0, diag / np.where(mean > 0, mean, 1.0), 1.0).astype(np.float32)
     lam, vec = np.linalg.eigh(M)             # ascending
     lam = lam[:, ::-1]
     vec = vec[:, :, ::-1]

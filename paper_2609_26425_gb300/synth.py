@@ -181,3 +181,23 @@ def bits(t: torch.Tensor) -> np.ndarray:
 def from_bits(a: np.ndarray) -> torch.Tensor:
     """numpy uint16 bf16 bit pattern -> bf16 CPU tensor."""
     return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+
+
+def hadamard_queries(H: int, d: int = 128) -> torch.Tensor:
+    """Queries along the rows of a Sylvester Hadamard matrix, [d][H][d] bf16.
+
+    Query n of head h is s_h(n) * had[n], with had the d x d matrix of +-1
+    built by repeated Kronecker doubling and s_h(n) = n + 1 for even heads,
+    d - n for odd heads (integers <= 256, exact in bf16).  The rows are
+    orthogonal, so the set's second moment has the rows as eigenvectors with
+    eigenvalues s_h(n)^2 and a constant diagonal.
+    """
+    had = torch.ones(1, 1, dtype=torch.float32)
+    while had.shape[0] < d:
+        had = torch.cat([torch.cat([had, had], 1), torch.cat([had, -had], 1)], 0)
+    n = torch.arange(d, dtype=torch.float32)
+    q = torch.empty(d, H, d, dtype=torch.float32)
+    for h in range(H):
+        s = n + 1 if h % 2 == 0 else d - n
+        q[:, h] = s[:, None] * had
+    return q.to(torch.bfloat16)

@@ -121,3 +121,48 @@ def test_query_stats_identities(orc):
         assert np.allclose(U[h].T @ U[h], np.eye(r), atol=1e-10)
         assert np.allclose(M[h] @ U[h], U[h] * lam[h, :r], atol=1e-8)
         assert np.all(np.diff(lam[h]) <= 1e-12)
+
+
+def test_query_stats_hadamard_closed_form(orc):
+    """Queries s_n * had_n along orthogonal +-1 rows (N = d = 128): by Eq. 6,
+    M = (1/N) sum_n s_n^2 had_n had_n^T, whose eigenvectors are the rows
+    had_n / sqrt(d) with eigenvalues s_n^2 (had_n^T had_n = d = N), and whose
+    diagonal is the constant mean(s^2), so Eq. 8 gives w = 1 exactly."""
+    H, d, r = 2, 128, 16
+    q = synth.hadamard_queries(H, d)
+    had = q[:, 0].float() / (torch.arange(d, dtype=torch.float32) + 1)[:, None]
+    M, w, U, lam = orc.query_stats(synth.bits(q), r)
+    assert np.all(w == 1.0)
+    for h in range(H):
+        s = np.arange(1, d + 1, dtype=np.float64) if h % 2 == 0 else np.arange(d, 0, -1, dtype=np.float64)
+        assert np.allclose(lam[h], np.sort(s ** 2)[::-1], rtol=1e-12)
+        top = np.argsort(-s, kind="stable")[:r]
+        for j in range(r):
+            ref = had[top[j]].double().numpy() / np.sqrt(d)
+            assert abs(abs(np.dot(U[h][:, j], ref)) - 1.0) < 1e-10
+
+
+def test_query_stats_diagonal_weights(orc):
+    """Query n = v_n e_n (one channel each): M = diag(v^2) / N, so Eq. 8 gives
+    w_c = v_c^2 / mean(v^2) and the eigenvectors are the unit channels in
+    decreasing v.  Values v_n = 1 + n/128 are exact in bf16."""
+    d, r = 128, 8
+    v = 1.0 + np.arange(d) / 128.0
+    q = np.zeros((d, 1, d), np.float32)
+    q[np.arange(d), 0, np.arange(d)] = v
+    qb = synth.bits(torch.from_numpy(q).to(torch.bfloat16))
+    M, w, U, lam = orc.query_stats(qb, r)
+    assert np.allclose(M[0], np.diag(v ** 2) / d, rtol=0, atol=1e-15)
+    assert np.allclose(w[0], v ** 2 / np.mean(v ** 2), rtol=1e-6)
+    for j in range(r):
+        assert abs(abs(U[0][d - 1 - j, j]) - 1.0) < 1e-12
+
+
+def test_query_stats_cold_start_and_zero_queries(orc):
+    """No Query seen: w = 1, U = 0 (App. C.3).  Only zero Queries: Eq. 8 is
+    0/0 and the head keeps the cold-start weights w = 1."""
+    H, d, r = 3, 128, 8
+    M, w, U, lam = orc.query_stats(np.zeros((0, H, d), np.uint16), r)
+    assert np.all(w == 1.0) and np.all(U == 0.0) and np.all(M == 0.0)
+    M, w, U, lam = orc.query_stats(np.zeros((5, H, d), np.uint16), r)
+    assert np.all(w == 1.0) and np.all(lam == 0.0)
