@@ -303,6 +303,8 @@ def run_gpu(args, wl, rank, world):
     e_ms = e0.elapsed_time(e1)
     e_ms = job_time_ms(e_ms, world, dev)
 
+    qs = query_stats_timing(qwm, cfg, qd, dev, max(3, min(args.steps, 20)), stream)
+
     pk = peaks()
     att_tflops = nums["attend_flops"] / (att_ms * 1e-3) / 1e12
     app_gbs = nums["append_bytes"] / (app_ms * 1e-3) / 1e9
@@ -332,8 +334,48 @@ def run_gpu(args, wl, rank, world):
         # when M <= 8 and M < C, a single kernel otherwise
         "gpu_launches": (1 + (2 if (M < C and M <= 8) else 1)) * args.steps,
         "clocks": clk,
+        "query_stats": {"update_ms": round(qs["update_ms"], 4),
+                        "update_gbs": round(qs["update_bytes"] / (qs["update_ms"] * 1e-3) / 1e9, 1),
+                        "update_frac_of_measured_hbm": round(
+                            qs["update_bytes"] / (qs["update_ms"] * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
+                        "update_algorithmic_bytes": qs["update_bytes"],
+                        "basis_ms": round(qs["basis_ms"], 4), "jacobi_sweeps": qs["sweeps"],
+                        "l2": "flushed (256 MB write) before each timed launch"},
     }
     return res
+
+
+def query_stats_timing(qwm, cfg, qd, dev, iters, stream):
+    """Chunk-boundary Query statistics: qwm_query_stats_update over the chunk's
+    Queries and qwm_query_basis (w and U_r), each timed alone with CUDA events
+    after an L2 flush (the Queries alone fit in L2)."""
+    import torch
+    st = qwm.QueryStats(cfg, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        st.update(qd)
+        st.basis()
+
+    def timed(fn):
+        ms = []
+        for _ in range(iters):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        return sum(ms) / len(ms)
+
+    upd = timed(lambda: st.update(qd))
+    bas = timed(lambda: st.basis())
+    status, _ = st.read()
+    if status:
+        raise RuntimeError(f"query statistics device status {status}")
+    H, d = cfg.num_heads, cfg.head_dim
+    nbytes = qd.numel() * qd.element_size() + 2 * H * d * d * 4
+    return {"update_ms": upd, "basis_ms": bas, "update_bytes": nbytes, "sweeps": st.sweeps()}
 
 
 # ---------------------------------------------------------------------------- CPU oracle

@@ -190,6 +190,53 @@ QWM_API qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* cache, con
                       const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,
                       void* out, float* lse, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Historical Query statistics and the principal Query basis, kept on the GPU
+ * (Sec. 4.1 Eq. 6 and 8, Sec. 4.2 Eq. 15; App. C.3 cold start; App. D.1: the
+ * per-head statistics are updated incrementally, the basis is recomputed at
+ * chunk boundaries, past Queries are not kept).  They produce the w and U
+ * arguments of qwm_quantize_append without a host round trip.
+ *
+ * A statistics buffer is caller-owned device memory of
+ * qwm_query_stats_bytes(cfg) bytes, 256-byte aligned:
+ *   byte 0    int32 device status word (QWM_OK or the first kernel error)
+ *   byte 8    uint64 Query count N_<t (tokens folded in so far)
+ *   byte 16   int32 Jacobi sweeps of the last qwm_query_basis (maximum over heads)
+ *   byte 256  fp32 sums S_h = sum over past Queries of q q^T, [H][d][d] row-major.
+ * --------------------------------------------------------------------------- */
+
+/* Size of a statistics buffer; 0 for an invalid configuration. */
+QWM_API size_t qwm_query_stats_bytes(const qwm_config* cfg);
+
+/* Zero a statistics buffer (no Query seen yet). */
+QWM_API qwm_status qwm_query_stats_reset(const qwm_config* cfg, void* stats, void* stream);
+
+/* Fold one chunk's Queries into the statistics (Eq. 6 numerator):
+ * S_h += sum_n q[n,h] q[n,h]^T and count += N.  q: bf16 [N][H][d], 16-byte
+ * aligned; N = 0 is a no-op.  Products are exact and accumulate in fp32 (tensor
+ * cores); the same inputs always give the same bits. */
+QWM_API qwm_status qwm_query_stats_update(const qwm_config* cfg, void* stats, const void* q, int64_t N,
+                                          void* stream);
+
+/* Channel weights and principal basis from the statistics, M_h = S_h / count.
+ *   w: fp32 [H][d], w_c = M_cc / mean_c' M_c'c' (Eq. 8); 1 for every channel
+ *      when count = 0 or the mean is 0 (App. C.3 cold start).
+ *   U: bf16 [H][d][r], r = cfg->psac_rank (not written when r = 0): the
+ *      eigenvectors of M_h for its r largest eigenvalues (Eq. 15), column j
+ *      for the j-th largest (equal eigenvalues in increasing index order), each
+ *      signed so that its largest-magnitude entry (the first such) is positive;
+ *      0 when count = 0.
+ *   eigenvalues: fp32 [H][d], all eigenvalues of M_h in decreasing order.
+ * Any of w, U, eigenvalues may be NULL.  The eigen-solver is cyclic Jacobi in
+ * fp32 on the whole 128 x 128 matrix, run until a sweep finds no off-diagonal
+ * entry above 2^-20 of the Frobenius norm (at most 30 sweeps). */
+QWM_API qwm_status qwm_query_basis(const qwm_config* cfg, const void* stats, float* w, void* U, float* eigenvalues,
+                                   void* stream);
+
+/* Synchronise `stream`, then read and clear the statistics' device status
+ * word (*status) and read the Query count (*count, may be NULL). */
+QWM_API qwm_status qwm_query_stats_read(void* stats, int32_t* status, int64_t* count, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -10,8 +10,10 @@ built, every call raises.
 Functions carry the C names:
   qwm_cache_bytes, qwm_fit_workspace_bytes, qwm_fit_centroids,
   qwm_fit_centroids_noalloc, qwm_quantize_append, qwm_attend,
-and ``Cache`` wraps qwm_cache_init / qwm_cache_free / qwm_cache_status /
-qwm_cache_layout / qwm_cache_chunk_info.
+``Cache`` wraps qwm_cache_init / qwm_cache_free / qwm_cache_status /
+qwm_cache_layout / qwm_cache_chunk_info, and ``QueryStats`` wraps a Query
+statistics buffer (qwm_query_stats_bytes / _reset / _update / _read and
+qwm_query_basis).
 """
 from __future__ import annotations
 
@@ -101,6 +103,16 @@ def lib():
             L.qwm_quantize_append.restype = ct.c_int
             L.qwm_attend.argtypes = [_CFG, _P, _P, ct.c_int64, _P, _P, ct.c_int64, ct.c_float, _P, _P, _P]
             L.qwm_attend.restype = ct.c_int
+            L.qwm_query_stats_bytes.argtypes = [_CFG]
+            L.qwm_query_stats_bytes.restype = ct.c_size_t
+            L.qwm_query_stats_reset.argtypes = [_CFG, _P, _P]
+            L.qwm_query_stats_reset.restype = ct.c_int
+            L.qwm_query_stats_update.argtypes = [_CFG, _P, _P, ct.c_int64, _P]
+            L.qwm_query_stats_update.restype = ct.c_int
+            L.qwm_query_basis.argtypes = [_CFG, _P, _P, _P, _P, _P]
+            L.qwm_query_basis.restype = ct.c_int
+            L.qwm_query_stats_read.argtypes = [_P, ct.POINTER(ct.c_int32), ct.POINTER(ct.c_int64), _P]
+            L.qwm_query_stats_read.restype = ct.c_int
             _lib = L
     return _lib
 
@@ -300,3 +312,63 @@ def qwm_attend(cfg: QwmConfig, cache: Cache, q, k_cur=None, v_cur=None, sm_scale
                                           _ptr(k_cur) if Ncur else None, _ptr(v_cur) if Ncur else None, Ncur,
                                           scale, _ptr(out), _ptr(lse), _stream()))
     return (out, lse) if (want_lse or lse is not None) else out
+
+
+# ------------------------------------------------------------------ Query statistics
+class QueryStats:
+    """Running per-head Query statistics in a torch-allocated device buffer
+    (qwm_query_stats_bytes bytes: a 256-byte header, then fp32 sums [H][d][d])."""
+
+    HEADER = 256
+
+    def __init__(self, cfg: QwmConfig, device=None):
+        self.cfg = cfg
+        nbytes = int(lib().qwm_query_stats_bytes(ct.byref(cfg)))
+        if nbytes == 0:
+            raise QwmError("qwm_query_stats_bytes", 2)
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+        self._raw = torch.empty(nbytes + 256, dtype=torch.uint8, device=dev)
+        off = (-self._raw.data_ptr()) % 256
+        self.buffer = self._raw[off:off + nbytes]
+        self.nbytes = nbytes
+        self.reset()
+
+    def reset(self):
+        _check("qwm_query_stats_reset", lib().qwm_query_stats_reset(ct.byref(self.cfg), _ptr(self.buffer),
+                                                                    _stream()))
+
+    @property
+    def sums(self) -> torch.Tensor:
+        """View of the fp32 sums S_h = sum q q^T, [H][d][d] (no copy)."""
+        H, d = self.cfg.num_heads, self.cfg.head_dim
+        return self.buffer[self.HEADER:].view(torch.float32).view(H, d, d)
+
+    def update(self, q):
+        """qwm_query_stats_update: fold one chunk's Queries q [N][H][d] (bf16) in."""
+        N = q.shape[0]
+        _bf16(q, (N, self.cfg.num_heads, self.cfg.head_dim), "q")
+        _check("qwm_query_stats_update", lib().qwm_query_stats_update(ct.byref(self.cfg), _ptr(self.buffer),
+                                                                      _ptr(q) if N else None, N, _stream()))
+
+    def basis(self, w=True, U=True, eigenvalues=False):
+        """qwm_query_basis: returns (w [H][d] fp32, U [H][d][r] bf16, eigenvalues
+        [H][d] fp32), each None when not requested (U also when r = 0)."""
+        H, d, r = self.cfg.num_heads, self.cfg.head_dim, self.cfg.psac_rank
+        dev = self.buffer.device
+        tw = torch.empty(H, d, dtype=torch.float32, device=dev) if w else None
+        tU = torch.empty(H, d, r, dtype=torch.bfloat16, device=dev) if (U and r > 0) else None
+        te = torch.empty(H, d, dtype=torch.float32, device=dev) if eigenvalues else None
+        _check("qwm_query_basis", lib().qwm_query_basis(ct.byref(self.cfg), _ptr(self.buffer), _ptr(tw),
+                                                        _ptr(tU), _ptr(te), _stream()))
+        return tw, tU, te
+
+    def read(self):
+        """(status, count): synchronises the stream and clears the status word."""
+        st, cnt = ct.c_int32(), ct.c_int64()
+        _check("qwm_query_stats_read", lib().qwm_query_stats_read(_ptr(self.buffer), ct.byref(st), ct.byref(cnt),
+                                                                  _stream()))
+        return st.value, cnt.value
+
+    def sweeps(self) -> int:
+        """Jacobi sweeps of the last basis computation (maximum over heads)."""
+        return int(self.buffer[16:20].view(torch.int32).item())

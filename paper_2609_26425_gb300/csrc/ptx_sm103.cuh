@@ -354,6 +354,24 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool b_mn_major, 
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// An MN-major operand that spans several 128-byte swizzle atoms along M (or
+// N): rows of the tile are K indices (128 bytes = 64 16-bit values of the
+// MN dimension each), 8-row K groups are 1024 bytes apart (stride field) and
+// consecutive 64-wide MN atoms are `mn_stride` bytes apart (leading field).
+__device__ __forceinline__ uint64_t desc_sw128_mn(uint32_t saddr, uint32_t mn_stride) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((mn_stride >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+// kind::f16 instruction descriptor with both operands MN-major (bits 15, 16).
+__host__ __device__ constexpr uint32_t idesc_f16_mn(int M, int N, bool bf16) {
+  return idesc_f16(M, N, true, bf16) | (1u << 15);
+}
+
 // D[tmem] (+)= A[smem] * B[smem]^T, one CTA, issued by one thread.
 __device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                           uint32_t accumulate) {
@@ -419,6 +437,15 @@ __device__ __forceinline__ uint32_t mapa(uint32_t saddr, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
+}
+// 16-byte load from the shared memory of a CTA of the cluster (address from mapa).
+__device__ __forceinline__ float4 ld_dsmem_f4(uint32_t cluster_addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(cluster_addr)
+               : "memory");
+  return v;
 }
 // Arrive (release, cluster scope) on an mbarrier given by its cluster address.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {

@@ -64,7 +64,11 @@ struct qwm_cache {
 
 namespace {
 
-bool supported(const qwm_config* c) {
+bool supported(const qwm_config* c) { return qwm::config_supported(c); }
+
+}  // namespace
+
+bool qwm::config_supported(const qwm_config* c) {
   if (c->num_heads < 1 || c->num_heads > 4096) return false;
   if (c->head_dim != qwm::kHeadDim) return false;
   if (c->group_size != 32 && c->group_size != 64) return false;
@@ -73,6 +77,8 @@ bool supported(const qwm_config* c) {
   if (c->num_candidates < 1 || c->kmeans_iters < 0) return false;
   return true;
 }
+
+namespace {
 
 bool same_shape(const qwm_config* a, const qwm_config* b) {
   return a->num_heads == b->num_heads && a->head_dim == b->head_dim && a->num_centroids == b->num_centroids &&

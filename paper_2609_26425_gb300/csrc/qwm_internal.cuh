@@ -73,6 +73,10 @@ __host__ __device__ inline int64_t head_offset(const Layout& L, int slot, int h)
   return kHeaderBytes + (int64_t)slot * L.slot_bytes + kSlotMetaBytes + (int64_t)h * L.head_bytes;
 }
 
+// The configurations the library accepts (head_dim 128, group size 32 or 64,
+// 1..256 centroids, PSAC rank 0/8/16/32, 1..4096 heads); qwm_api.cu.
+bool config_supported(const qwm_config* c);
+
 // ----------------------------------------------------------------------------
 // TMA tensor maps (host, qwm_api.cu).
 // Tokens x[N][H][128] (bf16): boxes of 64 channels x 1 head x box_rows tokens,
