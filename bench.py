@@ -304,6 +304,7 @@ def run_gpu(args, wl, rank, world):
     e_ms = job_time_ms(e_ms, world, dev)
 
     qs = query_stats_timing(qwm, cfg, qd, dev, max(3, min(args.steps, 20)), stream)
+    fit_ms = fit_timing(qwm, cfg, kd, vd, ws, dev, max(3, min(args.steps, 10)), stream)
 
     pk = peaks()
     att_tflops = nums["attend_flops"] / (att_ms * 1e-3) / 1e12
@@ -340,15 +341,38 @@ def run_gpu(args, wl, rank, world):
                             qs["update_bytes"] / (qs["update_ms"] * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
                         "update_algorithmic_bytes": qs["update_bytes"],
                         "basis_ms": round(qs["basis_ms"], 4), "jacobi_sweeps": qs["sweeps"],
-                        "l2": "flushed (256 MB write) before each timed launch"},
+                        "l2": "update: 4 rotating copies of q (192 MB); basis: 256 MB flush before each launch"},
+        # chunk boundary, not on the step: Lloyd k-means tables of the chunk's Keys and Values
+        "fit": {"ms_keys_and_values": round(fit_ms, 3), "kmeans_iters": wl.kmeans_iters,
+                "l2": "256 MB flush before each timed pair"},
     }
     return res
 
 
+def fit_timing(qwm, cfg, kd, vd, ws, dev, iters, stream):
+    """qwm_fit_centroids on the chunk's Keys and then its Values (the two
+    tables a chunk boundary fits), timed with CUDA events after an L2 flush."""
+    import torch
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    kc = qwm.qwm_fit_centroids(cfg, kd, workspace=ws)
+    vc = qwm.qwm_fit_centroids(cfg, vd, workspace=ws)
+    ms = []
+    for _ in range(iters):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        qwm.qwm_fit_centroids(cfg, kd, centroids=kc, workspace=ws)
+        qwm.qwm_fit_centroids(cfg, vd, centroids=vc, workspace=ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    return sum(ms) / len(ms)
+
+
 def query_stats_timing(qwm, cfg, qd, dev, iters, stream):
     """Chunk-boundary Query statistics: qwm_query_stats_update over the chunk's
-    Queries and qwm_query_basis (w and U_r), each timed alone with CUDA events
-    after an L2 flush (the Queries alone fit in L2)."""
+    Queries (back to back over inputs larger than L2) and qwm_query_basis (w and
+    U_r, each launch timed alone after an L2 flush), with CUDA events."""
     import torch
     st = qwm.QueryStats(cfg, device=dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
@@ -368,7 +392,18 @@ def query_stats_timing(qwm, cfg, qd, dev, iters, stream):
             ms.append(e0.elapsed_time(e1))
         return sum(ms) / len(ms)
 
-    upd = timed(lambda: st.update(qd))
+    # back-to-back updates over four copies of the chunk's Queries (192 MB
+    # together, more than L2), one event pair around the batch
+    qbufs = [qd.clone() for _ in range(4)]
+    flush.zero_()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(4 * iters):
+        st.update(qbufs[i % 4])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    upd = e0.elapsed_time(e1) / (4 * iters)
+    del qbufs
     bas = timed(lambda: st.basis())
     status, _ = st.read()
     if status:

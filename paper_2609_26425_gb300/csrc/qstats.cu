@@ -30,11 +30,12 @@ constexpr int kStatsHeader = 256;   // status word, count, sweeps; then the sums
 
 // ------------------------------------------------------------------ Gram sums
 constexpr int kGTok = 64;                        // tokens per stage
-constexpr int kGStages = 4;
+constexpr int kGStages = 6;
 constexpr int kGStage = kGTok * 256;             // two 8 KB boxes: channels [0,64) and [64,128)
 constexpr int kGThreads = 128;
 constexpr int kGBarOff = kGStages * kGStage;     // the [128][128] fp32 partial reuses the stages
-constexpr int kGSmem = kGBarOff + 128 + 1024;    // barriers + alignment slack
+constexpr int kGBarBytes = (2 * kGStages + 1) * 8;
+constexpr int kGSmem = kGBarOff + kGBarBytes + 8 + 1024;   // barriers, TMEM slot, flag, alignment slack
 static_assert(kGStages * kGStage >= 128 * 128 * 4, "partial sum buffer");
 
 __global__ void __launch_bounds__(kGThreads) gram_kernel(const __grid_constant__ CUtensorMap tm, uint8_t* stats,
@@ -42,9 +43,9 @@ __global__ void __launch_bounds__(kGThreads) gram_kernel(const __grid_constant__
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t base = smem_u32(sm);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kGBarOff);  // full[4], empty[4], done
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + kGBarOff + 72);
-  volatile int* s_err = reinterpret_cast<volatile int*>(sm + kGBarOff + 76);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kGBarOff);  // full[kGStages], empty[kGStages], done
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + kGBarOff + kGBarBytes);
+  volatile int* s_err = reinterpret_cast<volatile int*>(sm + kGBarOff + kGBarBytes + 4);
   auto bar = [&](int i) { return smem_u32(bars + i); };
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -66,6 +67,16 @@ __global__ void __launch_bounds__(kGThreads) gram_kernel(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tD = *tslot;
+
+  // rows [rank R, rank R + R) of the running sum S_h, which this CTA updates
+  // at the end: loaded now, while the tiles stream in
+  const int R = 128 / S;                                  // S in {1, 2, 4, 8}
+  float4* gS = reinterpret_cast<float4*>(stats + kStatsHeader) + (size_t)h * (128 * 32);
+  float4 acc[32];                                         // R * 32 / 128 <= 32 items per thread
+  const int nit = R / 4;
+#pragma unroll
+  for (int m = 0; m < 32; ++m)
+    if (m < nit) acc[m] = gS[rank * R * 32 + tid + 128 * m];
 
   if (warp == 0) {
     if (lane == 0) {  // TMA producer
@@ -134,23 +145,29 @@ __global__ void __launch_bounds__(kGThreads) gram_kernel(const __grid_constant__
   cluster_sync();
   tc_fence_after();
 
-  // ---- rows [rank R, rank R + R) of S_h: the running sum plus the partials
-  // of ranks 0, 1, ..., S-1, in that order
-  const int R = 128 / S;
-  float4* gS = reinterpret_cast<float4*>(stats + kStatsHeader) + (size_t)h * (128 * 32);
+  // ---- the running sum plus the partials of ranks 0, 1, ..., S-1, in that
+  // order; the loads of all ranks for a row are issued before the adds
   const uint32_t red_s = smem_u32(red);
-  for (int i = tid; i < R * 32; i += kGThreads) {
-    const int r = rank * R + (i >> 5), c4 = i & 31;
-    float4 acc = gS[r * 32 + c4];
-    const uint32_t off = red_s + (uint32_t)((r * 32 + (c4 ^ (r & 7))) * 16);
-    for (int src = 0; src < S; ++src) {
-      const float4 p = ld_dsmem_f4(mapa(off, (uint32_t)src));
-      acc.x += p.x;
-      acc.y += p.y;
-      acc.z += p.z;
-      acc.w += p.w;
+#pragma unroll
+  for (int m = 0; m < 32; ++m) {
+    if (m < nit) {
+      const int i = tid + 128 * m;
+      const int r = rank * R + (i >> 5), c4 = i & 31;
+      const uint32_t off = red_s + (uint32_t)((r * 32 + (c4 ^ (r & 7))) * 16);
+      float4 p[8];
+#pragma unroll
+      for (int src = 0; src < 8; ++src)
+        if (src < S) p[src] = ld_dsmem_f4(mapa(off, (uint32_t)src));
+#pragma unroll
+      for (int src = 0; src < 8; ++src)
+        if (src < S) {
+          acc[m].x += p[src].x;
+          acc[m].y += p[src].y;
+          acc[m].z += p[src].z;
+          acc[m].w += p[src].w;
+        }
+      gS[rank * R * 32 + i] = acc[m];
     }
-    gS[r * 32 + c4] = acc;
   }
   cluster_sync();  // no CTA leaves while its partial is still being read
   tc_fence_after();
@@ -168,7 +185,7 @@ constexpr int kMaxSweeps = 30;
 
 __host__ __device__ constexpr int basis_smem_bytes(int vrows) {
   return (128 + vrows) * kJs * 4   // A, V rows
-         + 6 * 64 * 4              // pair tables
+         + 4 * 64 * 4              // pair tables
          + 32 * 4 + 128 * 4        // reductions, eigenvalue order
          + 32 * 16 + 32 * 4;       // sign candidates, signs
 }
@@ -181,13 +198,11 @@ __global__ void __launch_bounds__(kJThreads, 1) basis_kernel(uint8_t* stats, flo
   const int VR = 128 / SJ;         // rows of V kept by this CTA: rank * VR + [0, VR)
   float* A = js;                   // [128][kJs], entry (i, j) at min(i,j) * kJs + max(i,j)
   float* V = A + 128 * kJs;        // [VR][kJs]
-  float* pc = V + VR * kJs;        // per pair: cos, sin, new a_ff, new a_gg, index f, index g
+  float* pc = V + VR * kJs;        // per pair: cos, sin, new a_ff, new a_gg
   float* psn = pc + 64;
   float* paf = psn + 64;
   float* pag = paf + 64;
-  int* pf = reinterpret_cast<int*>(pag + 64);
-  int* pg = pf + 64;
-  float* red = reinterpret_cast<float*>(pg + 64);
+  float* red = pag + 64;
   int* order = reinterpret_cast<int*>(red + 32);
   float4* cand = reinterpret_cast<float4*>(order + 128);
   float* sgn = reinterpret_cast<float*>(cand + 32);
@@ -236,6 +251,9 @@ __global__ void __launch_bounds__(kJThreads, 1) basis_kernel(uint8_t* stats, flo
   // ---- cyclic Jacobi sweeps; round rr pairs index 0 with 1 + rr and
   // 1 + (rr + k) % 127 with 1 + (rr - k) % 127 for k = 1..63, so each sweep
   // (127 rounds) meets every index pair once
+  auto wrap = [](int x) { return x >= 127 ? x - 127 : x; };   // x < 254
+  auto pair_f = [&](int rr, int k) { return k == 0 ? 0 : 1 + wrap(rr + k); };
+  auto pair_g = [&](int rr, int k) { return k == 0 ? 1 + rr : 1 + wrap(rr + 127 - k); };
   int sweeps = 0;
   for (; sweeps < kMaxSweeps; ++sweeps) {
     int any = 0;
@@ -243,22 +261,22 @@ __global__ void __launch_bounds__(kJThreads, 1) basis_kernel(uint8_t* stats, flo
     for (int rr = 0; rr < 127; ++rr) {
       int rot = 0;
       if (tid < 64) {
-        const int f = tid == 0 ? 0 : 1 + (rr + tid) % 127;
-        const int g = tid == 0 ? 1 + rr : 1 + (rr + 127 - tid) % 127;
+        const int f = pair_f(rr, tid), g = pair_g(rr, tid);
         const float aff = A[f * kJs + f], agg = A[g * kJs + g], afg = A[ut(f, g)];
         float c = 1.0f, s = 0.0f, nf = aff, ng = agg;
         if (fabsf(afg) > thr) {
-          // the rotation that zeroes a_fg: tan = sign(tau) / (|tau| + sqrt(1 + tau^2))
-          const float tau = (agg - aff) / (2.0f * afg);
-          const float t = copysignf(1.0f, tau) / (fabsf(tau) + sqrtf(fmaf(tau, tau, 1.0f)));
-          c = 1.0f / sqrtf(fmaf(t, t, 1.0f));
+          // the rotation that zeroes a_fg: tan = sign(tau) / (|tau| + sqrt(1 + tau^2)),
+          // |tau| <= 2^20 here; fast reciprocals: any (c, s) with c^2 + s^2 = 1
+          // to rounding is an orthogonal step, and a_fg is set to zero below
+          const float tau = __fdividef(agg - aff, 2.0f * afg);
+          const float q = fmaf(tau, tau, 1.0f);
+          const float t = __fdividef(copysignf(1.0f, tau), fabsf(tau) + q * rsqrtf(q));
+          c = rsqrtf(fmaf(t, t, 1.0f));
           s = t * c;
           nf = aff - t * afg;
           ng = agg + t * afg;
           rot = 1;
         }
-        pf[tid] = f;
-        pg[tid] = g;
         pc[tid] = c;
         psn[tid] = s;
         paf[tid] = nf;
@@ -268,44 +286,78 @@ __global__ void __launch_bounds__(kJThreads, 1) basis_kernel(uint8_t* stats, flo
       any = 1;
       // A <- J^T A J.  Off-diagonal 2 x 2 blocks {a, b}: warp-iteration b,
       // lanes a = (b + 1 + lane) % 64 (lane 31 only for b < 32), so each
-      // unordered pair of pairs is updated exactly once.
-#pragma unroll 1
-      for (int it = 0; it < 4; ++it) {
-        const int b = warp + 16 * it;
-        const int a = (b + 1 + lane) & 63;
-        if (lane == 31 && b >= 32) continue;
-        const float sa = psn[a], sb = psn[b];
-        if (sa == 0.0f && sb == 0.0f) continue;
-        const float ca = pc[a], cb = pc[b];
-        const int ia = ut(pf[a], pf[b]), ib = ut(pf[a], pg[b]), ic = ut(pg[a], pf[b]), id = ut(pg[a], pg[b]);
-        const float x00 = A[ia], x01 = A[ib], x10 = A[ic], x11 = A[id];
-        // columns of pair b, then rows of pair a
-        const float y00 = cb * x00 - sb * x01, y01 = sb * x00 + cb * x01;
-        const float y10 = cb * x10 - sb * x11, y11 = sb * x10 + cb * x11;
-        A[ia] = ca * y00 - sa * y10;
-        A[ic] = sa * y00 + ca * y10;
-        A[ib] = ca * y01 - sa * y11;
-        A[id] = sa * y01 + ca * y11;
+      // unordered pair of pairs is updated exactly once.  The four blocks of
+      // a thread are disjoint: all loads first, then the rotations.
+      {
+        int ix[4][4];
+        float cs[4][4], x[4][4];
+        bool act[4];
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+          const int b = warp + 16 * it;
+          const int a = (b + 1 + lane) & 63;
+          cs[it][0] = pc[a];
+          cs[it][1] = psn[a];
+          cs[it][2] = pc[b];
+          cs[it][3] = psn[b];
+          act[it] = !(lane == 31 && b >= 32) && (cs[it][1] != 0.0f || cs[it][3] != 0.0f);
+          const int fa = pair_f(rr, a), ga = pair_g(rr, a), fb = pair_f(rr, b), gb = pair_g(rr, b);
+          ix[it][0] = ut(fa, fb);
+          ix[it][1] = ut(fa, gb);
+          ix[it][2] = ut(ga, fb);
+          ix[it][3] = ut(ga, gb);
+        }
+#pragma unroll
+        for (int it = 0; it < 4; ++it)
+          if (act[it])
+#pragma unroll
+            for (int e = 0; e < 4; ++e) x[it][e] = A[ix[it][e]];
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+          if (!act[it]) continue;
+          const float ca = cs[it][0], sa = cs[it][1], cb = cs[it][2], sb = cs[it][3];
+          // columns of pair b, then rows of pair a
+          const float y00 = cb * x[it][0] - sb * x[it][1], y01 = sb * x[it][0] + cb * x[it][1];
+          const float y10 = cb * x[it][2] - sb * x[it][3], y11 = sb * x[it][2] + cb * x[it][3];
+          A[ix[it][0]] = ca * y00 - sa * y10;
+          A[ix[it][2]] = sa * y00 + ca * y10;
+          A[ix[it][1]] = ca * y01 - sa * y11;
+          A[ix[it][3]] = sa * y01 + ca * y11;
+        }
       }
       // the diagonal block of each rotated pair in closed form
       if (tid < 64 && psn[tid] != 0.0f) {
-        const int f = pf[tid], g = pg[tid];
+        const int f = pair_f(rr, tid), g = pair_g(rr, tid);
         A[f * kJs + f] = paf[tid];
         A[g * kJs + g] = pag[tid];
         A[ut(f, g)] = 0.0f;
       }
-      // V <- V J on this CTA's rows
-#pragma unroll 1
-      for (int it = 0; it < 4; ++it) {
-        const int b = warp + 16 * it;
-        const float sb = psn[b];
-        if (sb == 0.0f) continue;
-        const float cb = pc[b];
-        const int f = pf[b], g = pg[b];
+      // V <- V J on this CTA's rows (columns of four disjoint pairs per warp)
+      {
+        int vf[4], vg[4];
+        float vc[4], vs[4];
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+          const int b = warp + 16 * it;
+          vc[it] = pc[b];
+          vs[it] = psn[b];
+          vf[it] = pair_f(rr, b);
+          vg[it] = pair_g(rr, b);
+        }
         for (int i = lane; i < VR; i += 32) {
-          const float x = V[i * kJs + f], y = V[i * kJs + g];
-          V[i * kJs + f] = cb * x - sb * y;
-          V[i * kJs + g] = sb * x + cb * y;
+          float x[4], y[4];
+#pragma unroll
+          for (int it = 0; it < 4; ++it)
+            if (vs[it] != 0.0f) {
+              x[it] = V[i * kJs + vf[it]];
+              y[it] = V[i * kJs + vg[it]];
+            }
+#pragma unroll
+          for (int it = 0; it < 4; ++it)
+            if (vs[it] != 0.0f) {
+              V[i * kJs + vf[it]] = vc[it] * x[it] - vs[it] * y[it];
+              V[i * kJs + vg[it]] = vs[it] * x[it] + vc[it] * y[it];
+            }
         }
       }
       __syncthreads();
