@@ -126,8 +126,11 @@ QWM_API qwm_status qwm_cache_layout(const qwm_cache* cache, qwm_layout* out);
  * receives QWM_OK or the first error a kernel recorded (QWM_ERR_TIMEOUT). */
 QWM_API qwm_status qwm_cache_status(qwm_cache* cache, int32_t* status, void* stream);
 
-/* Scratch bytes qwm_fit_centroids needs for N tokens (fp32 centroids, fp64
- * member sums and counts); 0 for an invalid configuration. */
+/* Scratch bytes qwm_fit_centroids needs for N tokens; 0 for an invalid
+ * configuration.  With P = C rounded up to a multiple of 16 (at least 16),
+ * each part padded to 256 bytes: a 256-byte status word, fp32 centroids
+ * H*C*d*4, bf16 operand images H*P*512, norms H*P*4, H*4, counts and offsets
+ * 2*H*C*4, assignment H*N and member lists H*N*4. */
 QWM_API size_t qwm_fit_workspace_bytes(const qwm_config* cfg, int64_t N);
 
 /* k-means centroids of one chunk, per head (Sec. 2: centroid-residual form of
@@ -136,8 +139,12 @@ QWM_API size_t qwm_fit_workspace_bytes(const qwm_config* cfg, int64_t N);
  * Initial centroid j is token floor(j*N/C); each of kmeans_iters iterations
  * assigns every token to its Euclidean-nearest centroid (ties to the lower
  * index) and replaces each non-empty cluster's centroid by its member mean;
- * the result is rounded to bf16.  workspace: device scratch of at least
- * qwm_fit_workspace_bytes(cfg, N) bytes, 256-byte aligned. */
+ * the result is rounded to bf16.  The distance is the fp32 sum in channel
+ * order of the rounded squares of the rounded differences, the mean the fp32
+ * rounding of the fp64 mean: the tensor cores screen the centroids and every
+ * decision is taken on these exact values.  workspace: device scratch of at
+ * least qwm_fit_workspace_bytes(cfg, N) bytes, 256-byte aligned.  If a bounded
+ * wait inside a kernel runs out, every output centroid is NaN. */
 QWM_API qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, void* centroids,
                              void* workspace, size_t workspace_bytes, void* stream);
 
@@ -147,9 +154,8 @@ QWM_API qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64
  * whose device memory is reserved by its own pool and which must not call
  * cudaMalloc/cudaFree mid-generation (they can synchronise the device).  The
  * k-means scratch lives in a static 16 MiB device array that every GPU which
- * loads the library keeps until process exit; configurations needing more
- * (fp32 + fp64 + count scratch of H*C*(12*d + 4) bytes, 256-byte padded per
- * part) return QWM_ERR_CAPACITY.  Same arguments and results as
+ * loads the library keeps until process exit; calls needing more
+ * (qwm_fit_workspace_bytes(cfg, N) above 16 MiB) return QWM_ERR_CAPACITY.  Same arguments and results as
  * qwm_fit_centroids without the workspace.  The first call on a device looks
  * up the array's device address on the current device, so make that first
  * call before any stream capture.  All calls share the one array: calls whose

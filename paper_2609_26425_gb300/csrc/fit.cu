@@ -1,101 +1,480 @@
 // fit.cu -- k-means centroids of one chunk per head (Sec. 2: the
 // centroid-residual form of QVG with centroids kept in BF16, App. D.1).
 //
-// Lloyd iterations: initial centroid j = token floor(j*N/C); each iteration
-// assigns every token to its Euclidean-nearest centroid (distance summed in
-// channel order in fp32 with explicitly rounded operations, ties to the lower
-// index) and replaces each non-empty cluster by its member mean (member sums
-// accumulated in fp64, which is exact for bf16 members of ordinary range, so
-// the result does not depend on the order of the atomic adds).
+// Lloyd's algorithm with the arithmetic of its plain definition: initial
+// centroid j = token floor(j*N/C); each iteration assigns every token to its
+// Euclidean-nearest centroid, the distance being the fp32 sum in channel order
+// of the rounded squares of the rounded differences (ties to the lower
+// index), then replaces each non-empty cluster by the fp32 rounding of its
+// fp64 member mean; the result is rounded to bf16.  Per iteration:
+//
+//   fit_assign  (persistent, one CTA per SM, tcgen05).  A 128-token tile
+//     arrives by TMA and two MMAs per K step accumulate
+//     P = X mu_hi^T + X mu_lo^T in TMEM (mu_hi = bf16(mu), mu_lo =
+//     bf16(mu - mu_hi): mu to 2^-18 relative; bf16 x bf16 products are exact).
+//     With dt_j = |mu_j|^2 - 2 P_j, |dt_j + |x|^2 - d_j| stays below
+//     E = 2^-11 (|x|^2 + max_j |mu_j|^2) for the sequential fp32 distance d_j
+//     (operand split 2^-18, fp32 accumulation of 256 products 2^-15, the
+//     norms and the sequential sum's own rounding (d + 2) 2^-24, each relative
+//     to |x|^2 + |mu_j|^2, with margin).  Every centroid within 2E of the
+//     smallest dt is therefore a candidate for the exact argmin; a row with a
+//     single candidate is decided, the others (a few percent) are rescored
+//     with the sequential fp32 distance.
+//   fit_scatter (one CTA per head): counting sort of the tokens by cluster.
+//   fit_means   (one warp per centroid): exact fp64 member sums (bf16 values
+//     of ordinary range add exactly, so the order does not matter), the mean,
+//     and the next iteration's operand images and norm.
 #include <mutex>
 
+#include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
 
 namespace qwm {
 namespace {
 
-constexpr int FT = 128;  // tokens per assign CTA
+using namespace ptx;
 
-__global__ void fit_init_kernel(const FitArgs a) {
-  const int64_t n = (int64_t)a.H * a.C * a.d;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int c = (int)(i % a.d);
-    const int j = (int)((i / a.d) % a.C);
-    const int h = (int)(i / ((int64_t)a.d * a.C));
-    const int64_t src = ((int64_t)j * a.N) / a.C;
-    a.cent[i] = __bfloat162float(a.x[(src * a.H + h) * a.d + c]);
+constexpr int AT = 128;                       // tokens per tile = threads per assign CTA
+constexpr int kPairCap = 1024;                // (row, centroid) pairs rescored per tile
+constexpr int kRowCap = 8;                    // candidates listed per row
+constexpr int A_X = 0;                        // token tile: 2 x [128 rows][128 B] bf16
+constexpr int A_IMG = 32768;                  // operand images hi, lo: 2 x 2 x [Npad][128 B]
+constexpr int A_NRM = A_IMG + 131072;         // |mu_j|^2 [256]
+constexpr int A_PJ = A_NRM + 1024;            // pair (row << 16 | j) [kPairCap]
+constexpr int A_PD = A_PJ + kPairCap * 4;     // pair distance [kPairCap]
+constexpr int A_ROW = A_PD + kPairCap * 4;    // row: first slot << 16 | count (0xFFFF: full scan)
+constexpr int A_BAR = A_ROW + AT * 4;         // 3 mbarriers, pair counter, flag, TMEM slot
+constexpr int A_SMEM = A_BAR + 64 + 1024;
+
+// Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in two
+// 128-byte-swizzled blocks of `rows` rows x 64 two-byte elements.
+__device__ __forceinline__ int sw_off(int rows, int row, int ch) {
+  return (ch >> 3) * rows * 128 + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
+}
+
+// The sequential fp32 distance of the definition: channel order, the
+// difference, its square and the running sum each rounded on its own.
+__device__ float exact_dist(const uint8_t* sX, int row, const float* mu) {
+  float acc = 0.0f;
+#pragma unroll 2
+  for (int ch = 0; ch < 16; ++ch) {
+    const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
+    const float4 m0 = __ldg(reinterpret_cast<const float4*>(mu + ch * 8));
+    const float4 m1 = __ldg(reinterpret_cast<const float4*>(mu + ch * 8 + 4));
+    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+    const float ms[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float xe = (e & 1) ? __uint_as_float(xw[e >> 1] & 0xFFFF0000u) : __uint_as_float(xw[e >> 1] << 16);
+      const float t = __fsub_rn(xe, ms[e]);
+      acc = __fadd_rn(acc, __fmul_rn(t, t));
+    }
+  }
+  return acc;
+}
+
+// Operand images and norm of centroid j of head h from its fp32 row (one
+// warp, lane = channels 4 lane .. 4 lane + 3).
+__device__ __forceinline__ void emit_row(const FitArgs& a, int h, int j, float4 m, int lane) {
+  const int c0 = 4 * lane;
+  const __nv_bfloat162 h01 = __floats2bfloat162_rn(m.x, m.y), h23 = __floats2bfloat162_rn(m.z, m.w);
+  const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+  const __nv_bfloat162 l01 = __floats2bfloat162_rn(m.x - f01.x, m.y - f01.y);
+  const __nv_bfloat162 l23 = __floats2bfloat162_rn(m.z - f23.x, m.w - f23.y);
+  const size_t off = (size_t)sw_off(a.Npad, j, c0 >> 3) + (size_t)(c0 & 7) * 2;
+  uint8_t* hi = a.img + (size_t)h * 2 * a.Npad * 256;
+  uint8_t* lo = hi + (size_t)a.Npad * 256;
+  *reinterpret_cast<uint2*>(hi + off) =
+      make_uint2(*reinterpret_cast<const uint32_t*>(&h01), *reinterpret_cast<const uint32_t*>(&h23));
+  *reinterpret_cast<uint2*>(lo + off) =
+      make_uint2(*reinterpret_cast<const uint32_t*>(&l01), *reinterpret_cast<const uint32_t*>(&l23));
+  float n2 = fmaf(m.x, m.x, fmaf(m.y, m.y, fmaf(m.z, m.z, m.w * m.w)));
+#pragma unroll
+  for (int o = 16; o; o >>= 1) n2 += __shfl_xor_sync(0xFFFFFFFFu, n2, o);
+  if (lane == 0) {
+    a.nrm[(size_t)h * a.Npad + j] = n2;
+    atomicMax(a.nmax + h, __float_as_uint(n2));  // n2 >= 0: the bits order like the values
   }
 }
 
-__global__ void __launch_bounds__(FT) fit_assign_kernel(const FitArgs a) {
-  extern __shared__ float sx[];  // [FT][d + 1]
-  const int h = blockIdx.y;
-  const int d = a.d, C = a.C;
-  const int64_t t0 = (int64_t)blockIdx.x * FT;
-  const int ld = d + 1;
-  for (int i = threadIdx.x; i < FT * d; i += FT) {
-    const int ti = i / d, c = i % d;
-    const int64_t t = t0 + ti;
-    sx[ti * ld + c] = t < a.N ? __bfloat162float(a.x[(t * a.H + h) * d + c]) : 0.0f;
+// Initial centroids (token floor(j N / C)) and their images; padding rows
+// j in [C, Npad) get zero images and norm.  One warp per (head, row).
+__global__ void __launch_bounds__(512) fit_prep(const FitArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= (int64_t)a.H * a.Npad) return;
+  const int h = (int)(w / a.Npad), j = (int)(w % a.Npad);
+  if (j >= a.C) {
+    const size_t off = (size_t)sw_off(a.Npad, j, lane >> 1) + (size_t)(lane & 1) * 8;
+    uint8_t* hi = a.img + (size_t)h * 2 * a.Npad * 256;
+    *reinterpret_cast<uint2*>(hi + off) = make_uint2(0, 0);
+    *reinterpret_cast<uint2*>(hi + (size_t)a.Npad * 256 + off) = make_uint2(0, 0);
+    if (lane == 0) a.nrm[(size_t)h * a.Npad + j] = 0.0f;
+    return;
+  }
+  const int64_t src = ((int64_t)j * a.N) / a.C;
+  const uint2 xv = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)src * a.H + h) * 128 + 4 * lane));
+  const float4 m = make_float4(__uint_as_float(xv.x << 16), __uint_as_float(xv.x & 0xFFFF0000u),
+                               __uint_as_float(xv.y << 16), __uint_as_float(xv.y & 0xFFFF0000u));
+  reinterpret_cast<float4*>(a.cent + ((size_t)h * a.C + j) * 128)[lane] = m;
+  emit_row(a, h, j, m, lane);
+}
+
+// Assignment of every token (see the file comment).  Units are (head, tile)
+// in head-major order, split into contiguous runs over the CTAs, so a CTA
+// loads the images of a head once per run.
+__global__ void __launch_bounds__(AT, 1)
+    fit_assign(const FitArgs a, const __grid_constant__ CUtensorMap tm, int tiles, int units) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int tid = threadIdx.x, warp = tid >> 5, row = tid;
+  const int C = a.C, Npad = a.Npad;
+  uint8_t* sX = sm + A_X;
+  const float* sNrm = reinterpret_cast<const float*>(sm + A_NRM);
+  uint32_t* sPJ = reinterpret_cast<uint32_t*>(sm + A_PJ);
+  float* sPD = reinterpret_cast<float*>(sm + A_PD);
+  uint32_t* sRow = reinterpret_cast<uint32_t*>(sm + A_ROW);
+  const uint32_t bar_tma = smem_u32(sm + A_BAR), bar_img = bar_tma + 8, bar_mma = bar_tma + 16;
+  int* s_np = reinterpret_cast<int*>(sm + A_BAR + 24);
+  volatile int* s_err = reinterpret_cast<volatile int*>(sm + A_BAR + 28);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + A_BAR + 32);
+  uint32_t ncols = 32;
+  while ((int)ncols < Npad) ncols <<= 1;
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tslot), ncols);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    mbar_init(bar_tma, 1);
+    mbar_init(bar_img, 1);
+    mbar_init(bar_mma, 1);
+    fence_mbar_init();
+    *s_np = 0;
+    *s_err = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tD = *tslot;
+  const uint32_t lrow = (uint32_t)(warp * 32) << 16;
+  const int nchunk = (Npad + 31) >> 5;
+  const uint32_t id = idesc_f16(128, Npad, false, true);
+
+  const int u0 = (int)((int64_t)blockIdx.x * units / gridDim.x);
+  const int u1 = (int)((int64_t)(blockIdx.x + 1) * units / gridDim.x);
+  uint32_t ph_tma = 0, ph_img = 0, ph_mma = 0;
+  int cur_h = -1;
+  float nmx = 0.0f;
+  for (int u = u0; u < u1; ++u) {
+    const int h = u / tiles, tile = u - h * tiles;
+    if (h != cur_h) {  // this head's operand images and norms (earlier MMAs have completed)
+      if (tid == 0) {
+        const uint32_t ib = (uint32_t)Npad * 512u;
+        mbar_arrive_expect_tx(bar_img, ib + (uint32_t)Npad * 4u);
+        bulk_g2s(smem_u32(sm + A_IMG), a.img + (size_t)h * ib, ib, bar_img);
+        bulk_g2s(smem_u32(sm + A_NRM), a.nrm + (size_t)h * Npad, (uint32_t)Npad * 4u, bar_img);
+      }
+      if (!mbar_wait(bar_img, ph_img)) *s_err = 1;
+      ph_img ^= 1;
+      nmx = __uint_as_float(a.nmax[h]);
+      cur_h = h;
+    }
+    if (tid == 0) {
+      mbar_arrive_expect_tx(bar_tma, 32768);
+      tma_load_3d(smem_u32(sX), &tm, 0, h, tile * 128, bar_tma);
+      tma_load_3d(smem_u32(sX + 16384), &tm, 64, h, tile * 128, bar_tma);
+    }
+    if (!mbar_wait(bar_tma, ph_tma)) *s_err = 1;
+    ph_tma ^= 1;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (*s_err) break;
+    if (tid == 0) {
+      const uint32_t aX = smem_u32(sX), aI = smem_u32(sm + A_IMG);
+#pragma unroll
+      for (int half = 0; half < 2; ++half)
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            umma_ss(tD, desc_sw128(aX + kb * 16384 + ks * 32),
+                    desc_sw128(aI + half * Npad * 256 + kb * Npad * 128 + ks * 32), id, (half | kb | ks) != 0);
+      umma_commit(bar_mma);
+    }
+    // |x|^2 of this row while the MMAs run (any order: it only sizes E)
+    float kx = 0.0f;
+#pragma unroll 4
+    for (int ch = 0; ch < 16; ++ch) {
+      const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
+      const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const float x0 = __uint_as_float(xw[p] << 16), x1 = __uint_as_float(xw[p] & 0xFFFF0000u);
+        kx = fmaf(x0, x0, fmaf(x1, x1, kx));
+      }
+    }
+    bool ok = mbar_wait(bar_mma, ph_mma);
+    ph_mma ^= 1;
+    ok = __all_sync(0xFFFFFFFFu, ok);
+    tc_fence_after();
+    if (!ok) *s_err = 1;
+
+    // ---- smallest dt, then the candidates within 2E of it
+    float mn = INFINITY;
+    if (ok) {
+#pragma unroll 1
+      for (int cb = 0; cb < nchunk; ++cb) {
+        float v[32];
+        tmem_ld32(tD + lrow + cb * 32, v);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const int j = cb * 32 + e;
+          const float dt = j < C ? fmaf(-2.0f, v[e], sNrm[j]) : INFINITY;
+          mn = fminf(mn, dt);
+        }
+      }
+    }
+    const float thr = mn + 2.0f * ldexpf(kx + nmx, -11);
+    const int64_t n = (int64_t)tile * 128 + row;
+    const bool valid = n < a.N;
+    bool full = !(thr < INFINITY);
+    int cnt = 0;
+    int cj[kRowCap];
+#pragma unroll
+    for (int s2 = 0; s2 < kRowCap; ++s2) cj[s2] = 0;
+    if (ok) {
+#pragma unroll 1
+      for (int cb = 0; cb < nchunk; ++cb) {
+        float v[32];
+        tmem_ld32(tD + lrow + cb * 32, v);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const int j = cb * 32 + e;
+          if (j < C && fmaf(-2.0f, v[e], sNrm[j]) <= thr) {
+#pragma unroll
+            for (int s2 = 0; s2 < kRowCap; ++s2)
+              if (s2 == cnt) cj[s2] = j;
+            ++cnt;
+          }
+        }
+      }
+    }
+    full = full || cnt > kRowCap || cnt == 0;
+    uint32_t rinfo = 0;
+    if (valid && ok && !full && cnt > 1) {
+      const int base = atomicAdd(s_np, cnt);
+      if (base + cnt <= kPairCap) {
+#pragma unroll
+        for (int s2 = 0; s2 < kRowCap; ++s2)
+          if (s2 < cnt) sPJ[base + s2] = ((uint32_t)row << 16) | (uint32_t)cj[s2];
+        rinfo = ((uint32_t)base << 16) | (uint32_t)cnt;
+      } else {
+        full = true;
+      }
+    }
+    if (full) rinfo = 0xFFFFu;
+    sRow[row] = rinfo;
+    tc_fence_before();
+    __syncthreads();
+    // ---- exact rescoring of the listed pairs, spread over the CTA
+    const int np = min(*s_np, kPairCap);
+    const float* muh = a.cent + (size_t)cur_h * C * 128;
+    for (int p = tid; p < np; p += AT) {
+      const uint32_t pj = sPJ[p];
+      sPD[p] = exact_dist(sX, (int)(pj >> 16), muh + (size_t)(pj & 0xFFFFu) * 128);
+    }
+    __syncthreads();
+    if (valid && ok) {
+      int best = cj[0];
+      if (rinfo == 0xFFFFu) {  // every centroid, sequentially (non-finite rows, crowded bands)
+        float bd = 0.0f;
+        for (int j = 0; j < C; ++j) {
+          const float dj = exact_dist(sX, row, muh + (size_t)j * 128);
+          if (j == 0 || dj < bd) {
+            bd = dj;
+            best = j;
+          }
+        }
+      } else if (rinfo != 0) {
+        const int base = (int)(rinfo >> 16), c2 = (int)(rinfo & 0xFFFFu);
+        float bd = sPD[base];
+        best = (int)(sPJ[base] & 0xFFFFu);
+        for (int s2 = 1; s2 < c2; ++s2)
+          if (sPD[base + s2] < bd) {  // ascending j: the lower index keeps a tie
+            bd = sPD[base + s2];
+            best = (int)(sPJ[base + s2] & 0xFFFFu);
+          }
+      }
+      a.asg[(size_t)cur_h * a.N + n] = (uint8_t)best;
+      atomicAdd(a.counts + (size_t)cur_h * C + best, 1);
+    }
+    fence_proxy_async_smem();  // generic reads of the tile before the next copy overwrites it
+    __syncthreads();
+    if (tid == 0) *s_np = 0;
+  }
+  if (tid == 0 && *s_err) atomicCAS(a.status, 0, (int)QWM_ERR_TIMEOUT);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tD, ncols);
+  }
+}
+
+// Counting sort of one head's tokens by cluster: offsets from the counts,
+// then each token to a slot of its cluster (any order within a cluster).
+__global__ void __launch_bounds__(1024) fit_scatter(const FitArgs a) {
+  __shared__ int s_off[256], s_cur[256];
+  const int h = blockIdx.x, tid = threadIdx.x, C = a.C;
+  if (tid == 0) {
+    int o = 0;
+    for (int j = 0; j < C; ++j) {
+      s_off[j] = o;
+      o += a.counts[(size_t)h * C + j];
+    }
+    a.nmax[h] = 0u;  // rebuilt by fit_means
   }
   __syncthreads();
-  const int64_t t = t0 + threadIdx.x;
-  if (t >= a.N) return;
-  const float* xr = sx + threadIdx.x * ld;
-  const float* mu = a.cent + (size_t)h * C * d;
-  float best = 0.0f;
-  int bj = -1;
-  for (int j = 0; j < C; ++j) {
-    const float* m = mu + (size_t)j * d;
-    float acc = 0.0f;
-    for (int c = 0; c < d; ++c) {
-      const float tt = __fsub_rn(xr[c], __ldg(m + c));
-      acc = __fadd_rn(acc, __fmul_rn(tt, tt));
+  if (tid < C) {
+    a.offs[(size_t)h * C + tid] = s_off[tid];
+    s_cur[tid] = 0;
+  }
+  __syncthreads();
+  const uint8_t* asg = a.asg + (size_t)h * a.N;
+  int32_t* lst = a.list + (size_t)h * a.N;
+  // (the bounds checks only matter after a timed-out assignment left stale entries)
+  for (int64_t n = tid; n < a.N; n += blockDim.x) {
+    const int j = asg[n];
+    if (j < C) {
+      const int pos = s_off[j] + atomicAdd(&s_cur[j], 1);
+      if (pos < a.N) lst[pos] = (int32_t)n;
     }
-    if (bj < 0 || acc < best) { best = acc; bj = j; }
-  }
-  atomicAdd(a.counts + (size_t)h * C + bj, 1u);
-  double* sum = a.sums + ((size_t)h * C + bj) * d;
-  for (int c = 0; c < d; ++c) atomicAdd(sum + c, (double)xr[c]);
-}
-
-__global__ void fit_update_kernel(const FitArgs a) {
-  const int64_t n = (int64_t)a.H * a.C * a.d;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const uint32_t cnt = a.counts[i / a.d];
-    if (cnt) a.cent[i] = __double2float_rn(__ddiv_rn(a.sums[i], (double)cnt));
   }
 }
 
-__global__ void fit_out_kernel(const FitArgs a) {
-  const int64_t n = (int64_t)a.H * a.C * a.d;
+// New centroid j of head h: the fp32 rounding of the fp64 member mean (kept
+// when the cluster is empty); then its images and norm.  One warp each, lane =
+// four channels; the member rows are read four at a time.
+__global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= (int64_t)a.H * a.C) return;
+  const int h = (int)(w / a.C), j = (int)(w % a.C);
+  const int cnt = a.counts[w], base = a.offs[w];
+  float4* cr = reinterpret_cast<float4*>(a.cent + (size_t)w * 128) + lane;
+  float4 m;
+  if (cnt > 0) {
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    const int32_t* lst = a.list + (size_t)h * a.N + (base < a.N ? base : 0);
+    for (int i = 0; i < cnt; i += 4) {
+      uint2 xv[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        xv[k] = make_uint2(0, 0);
+        const int64_t tok = i + k < cnt ? (int64_t)lst[i + k] : -1;
+        if (tok >= 0 && tok < a.N)  // always, unless a timed-out assignment left stale lists
+          xv[k] = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)tok * a.H + h) * 128 + 4 * lane));
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if (i + k < cnt) {
+          s0 += (double)__uint_as_float(xv[k].x << 16);
+          s1 += (double)__uint_as_float(xv[k].x & 0xFFFF0000u);
+          s2 += (double)__uint_as_float(xv[k].y << 16);
+          s3 += (double)__uint_as_float(xv[k].y & 0xFFFF0000u);
+        }
+    }
+    const double dc = (double)cnt;
+    m = make_float4(__double2float_rn(__ddiv_rn(s0, dc)), __double2float_rn(__ddiv_rn(s1, dc)),
+                    __double2float_rn(__ddiv_rn(s2, dc)), __double2float_rn(__ddiv_rn(s3, dc)));
+    *cr = m;
+  } else {
+    m = *cr;
+  }
+  emit_row(a, h, j, m, lane);
+  __syncwarp();
+  if (lane == 0) a.counts[w] = 0;  // ready for the next assignment
+}
+
+// bf16 output; NaN everywhere if a wait inside the assignment ran out.
+__global__ void fit_out(const FitArgs a) {
+  const int64_t n = (int64_t)a.H * a.C * 128;
+  const bool bad = *a.status != 0;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-    a.out[i] = __float2bfloat16_rn(a.cent[i]);
+    a.out[i] = bad ? __float2bfloat16_rn(NAN) : __float2bfloat16_rn(a.cent[i]);
+}
+
+int sm_count() {
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) !=
+                                                 cudaSuccess || nsm < 1)
+    return 1;
+  return nsm;
 }
 
 }  // namespace
 
-size_t fit_workspace_bytes(int H, int d, int C) {
-  const size_t hcd = (size_t)H * C * d;
-  return (size_t)round_up(hcd * 4, 256) + (size_t)round_up(hcd * 8, 256) + (size_t)round_up((size_t)H * C * 4, 256);
+static int npad_of(int C) { return C < 16 ? 16 : (C + 15) & ~15; }
+
+size_t fit_workspace_bytes(int H, int d, int C, int64_t N) {
+  const int Np = npad_of(C);
+  size_t b = 256;                                               // status
+  b += (size_t)round_up((int64_t)H * C * d * 4, 256);           // cent
+  b += (size_t)round_up((int64_t)H * Np * 512, 256);            // images
+  b += (size_t)round_up((int64_t)H * Np * 4, 256);              // norms
+  b += (size_t)round_up((int64_t)H * 4, 256);                   // largest norm
+  b += 2 * (size_t)round_up((int64_t)H * C * 4, 256);           // counts, offsets
+  b += (size_t)round_up((int64_t)H * N, 256);                   // assignment
+  b += (size_t)round_up((int64_t)H * N * 4, 256);               // member lists
+  return b;
+}
+
+void fit_carve(FitArgs& a, uint8_t* ws) {
+  a.Npad = npad_of(a.C);
+  uint8_t* p = ws;
+  auto take = [&](int64_t bytes) {
+    uint8_t* q = p;
+    p += round_up(bytes, 256);
+    return q;
+  };
+  a.status = reinterpret_cast<int32_t*>(take(256));
+  a.cent = reinterpret_cast<float*>(take((int64_t)a.H * a.C * a.d * 4));
+  a.img = take((int64_t)a.H * a.Npad * 512);
+  a.nrm = reinterpret_cast<float*>(take((int64_t)a.H * a.Npad * 4));
+  a.nmax = reinterpret_cast<uint32_t*>(take((int64_t)a.H * 4));
+  a.counts = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
+  a.offs = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
+  a.asg = take((int64_t)a.H * a.N);
+  a.list = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.N * 4));
 }
 
 cudaError_t launch_fit(const FitArgs& a, cudaStream_t st) {
-  const int64_t n = (int64_t)a.H * a.C * a.d;
-  const int eb = 256;
-  const unsigned eg = (unsigned)((n + eb - 1) / eb < 4096 ? (n + eb - 1) / eb : 4096);
-  fit_init_kernel<<<eg, eb, 0, st>>>(a);
-  const size_t smem = (size_t)FT * (a.d + 1) * sizeof(float);
-  cudaError_t e = cudaFuncSetAttribute(fit_assign_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)((a.N + FT - 1) / FT), (unsigned)a.H);
-  for (int it = 0; it < a.iters; ++it) {
-    if ((e = cudaMemsetAsync(a.sums, 0, (size_t)n * sizeof(double), st)) != cudaSuccess) return e;
-    if ((e = cudaMemsetAsync(a.counts, 0, (size_t)a.H * a.C * sizeof(uint32_t), st)) != cudaSuccess) return e;
-    fit_assign_kernel<<<grid, FT, smem, st>>>(a);
-    fit_update_kernel<<<eg, eb, 0, st>>>(a);
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(a.status, 0, 4, st)) != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(a.nmax, 0, (size_t)a.H * 4, st)) != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(a.counts, 0, (size_t)a.H * a.C * 4, st)) != cudaSuccess) return e;
+  const int64_t prep_warps = (int64_t)a.H * a.Npad;
+  fit_prep<<<(unsigned)((prep_warps + 15) / 16), 512, 0, st>>>(a);
+  if (a.iters > 0) {
+    CUtensorMap tm;
+    if (!make_token_map(&tm, a.x, a.N, a.H, 128)) return cudaErrorInvalidValue;
+    if ((e = cudaFuncSetAttribute(fit_assign, cudaFuncAttributeMaxDynamicSharedMemorySize, A_SMEM)) != cudaSuccess)
+      return e;
+    const int tiles = (int)((a.N + 127) / 128);
+    const int units = a.H * tiles;
+    const int grid = units < sm_count() ? units : sm_count();
+    const int64_t mean_warps = (int64_t)a.H * a.C;
+    for (int it = 0; it < a.iters; ++it) {
+      fit_assign<<<grid, AT, A_SMEM, st>>>(a, tm, tiles, units);
+      fit_scatter<<<a.H, 1024, 0, st>>>(a);
+      fit_means<<<(unsigned)((mean_warps + 15) / 16), 512, 0, st>>>(a);
+    }
   }
-  fit_out_kernel<<<eg, eb, 0, st>>>(a);
+  const int64_t n = (int64_t)a.H * a.C * a.d;
+  const unsigned og = (unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  fit_out<<<og, 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -111,8 +490,8 @@ namespace qwm {
 // inference engine whose device memory is already reserved by its own pool
 // and which must not call cudaMalloc/cudaFree in the middle of generation
 // (those calls can synchronise the whole device).  For them the k-means
-// scratch (fp32 centroids, fp64 member sums, member counts) lives in this
-// file-scope device array instead.
+// scratch (fp32 centroids, MMA operand images, norms, counts, assignment and
+// member lists) lives in this file-scope device array instead.
 // ----------------------------------------------------------------------------
 namespace {
 
@@ -141,7 +520,7 @@ extern "C" QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, c
   if (N > (int64_t)1 << 31) return QWM_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(x) & 15u) || (reinterpret_cast<uintptr_t>(centroids) & 15u))
     return QWM_ERR_INVALID_ARG;
-  const size_t need = fit_workspace_bytes(cfg->num_heads, cfg->head_dim, cfg->num_centroids);
+  const size_t need = fit_workspace_bytes(cfg->num_heads, cfg->head_dim, cfg->num_centroids, N);
   if (need > kNoAllocFitScratchBytes) return QWM_ERR_CAPACITY;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return QWM_ERR_CUDA;
@@ -163,13 +542,10 @@ extern "C" QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, c
   a.N = N;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.out = static_cast<__nv_bfloat16*>(centroids);
-  const size_t hcd = (size_t)a.H * a.C * a.d;
-  a.cent = reinterpret_cast<float*>(ws);
-  a.sums = reinterpret_cast<double*>(ws + round_up(hcd * 4, 256));
-  a.counts = reinterpret_cast<uint32_t*>(ws + round_up(hcd * 4, 256) + round_up(hcd * 8, 256));
-  // launch_fit writes every centroid before reading it and clears the sums
-  // and counts before each iteration, so nothing depends on what an earlier
-  // call left in the array.
+  fit_carve(a, ws);
+  // launch_fit clears the status word, the counts and the largest norms and
+  // writes every centroid, image and norm before reading it, so nothing
+  // depends on what an earlier call left in the array.
   return launch_fit(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
 }
 

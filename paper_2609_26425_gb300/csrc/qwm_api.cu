@@ -187,7 +187,7 @@ qwm_status qwm_cache_status(qwm_cache* c, int32_t* status, void* stream) {
 
 size_t qwm_fit_workspace_bytes(const qwm_config* cfg, int64_t N) {
   if (!cfg || !supported(cfg) || N < 1) return 0;
-  return qwm::fit_workspace_bytes(cfg->num_heads, cfg->head_dim, cfg->num_centroids);
+  return qwm::fit_workspace_bytes(cfg->num_heads, cfg->head_dim, cfg->num_centroids, N);
 }
 
 qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, void* centroids, void* workspace,
@@ -203,11 +203,7 @@ qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, vo
   a.N = N;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.out = static_cast<__nv_bfloat16*>(centroids);
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  size_t hcd = (size_t)a.H * a.C * a.d;
-  a.cent = reinterpret_cast<float*>(ws);
-  a.sums = reinterpret_cast<double*>(ws + qwm::round_up(hcd * 4, 256));
-  a.counts = reinterpret_cast<uint32_t*>(ws + qwm::round_up(hcd * 4, 256) + qwm::round_up(hcd * 8, 256));
+  qwm::fit_carve(a, static_cast<uint8_t*>(workspace));
   return qwm::launch_fit(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
 }
 

@@ -126,15 +126,25 @@ struct AttendArgs {
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t s);
 
 struct FitArgs {
-  int H, d, C, iters;
+  int H, d, C, iters, Npad;    // Npad: C rounded up to a multiple of 16 (MMA width)
   int64_t N;
   const __nv_bfloat16* x;      // [N][H][d]
   __nv_bfloat16* out;          // [H][C][d]
-  float* cent;                 // workspace: [H][C][d] fp32
-  double* sums;                // workspace: [H][C][d] fp64
-  uint32_t* counts;            // workspace: [H][C]
+  // workspace (FitWorkspace carves it)
+  int32_t* status;             // device status word (a bounded wait that ran out)
+  float* cent;                 // [H][C][d] fp32 centroids
+  uint8_t* img;                // [H][2][Npad * 256] bf16 MMA operand images: hi, lo
+  float* nrm;                  // [H][Npad] squared centroid norms
+  uint32_t* nmax;              // [H] largest squared norm (fp32 bits)
+  int32_t* counts;             // [H][C] members per cluster
+  int32_t* offs;               // [H][C] first member slot
+  uint8_t* asg;                // [H][N] assignment
+  int32_t* list;               // [H][N] member token indices grouped by cluster
 };
-size_t fit_workspace_bytes(int H, int d, int C);
+// Byte size of the k-means workspace for H heads of N tokens and C centroids
+// (head_dim 128), and the carving of a workspace into FitArgs.
+size_t fit_workspace_bytes(int H, int d, int C, int64_t N);
+void fit_carve(FitArgs& a, uint8_t* ws);
 cudaError_t launch_fit(const FitArgs& a, cudaStream_t s);
 
 }  // namespace qwm

@@ -74,4 +74,6 @@ def test_unsupported_shapes_size_to_zero(qlib):
     assert qlib.qwm_cache_bytes(qlib.config(4, 64, psac_rank=12), 100, 2) == 0
     assert qlib.qwm_cache_bytes(qlib.config(4, 64), 100, 257) == 0
     assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 0) == 0
-    assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 10) >= 4 * 64 * 128 * 12
+    # centroids H*C*d*4, operand images H*P*512 (P = C rounded to 16), assignment and lists H*N*5
+    assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 10) >= 4 * 64 * 128 * 4 + 4 * 64 * 512 + 4 * 10 * 5
+    assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 20000) >= 4 * 64 * 128 * 4 + 4 * 64 * 512 + 4 * 20000 * 5

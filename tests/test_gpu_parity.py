@@ -105,31 +105,40 @@ def test_append_parity_fitted_tables():
     run_append_case(4, 880, 64, 32, 16, 4, True, True, seed=7, fit_iters=10)
 
 
-def test_fit_parity():
-    H, N, C, iters = 4, 880, 64, 10
-    _, k, _ = make_chunk(11, N, H)
+@pytest.mark.parametrize("H,N,C,iters", [
+    (4, 880, 64, 10),      # the single-layer workload's table
+    (3, 130, 4, 5),        # fewer centroids than one MMA column block
+    (2, 1000, 100, 4),     # C not a multiple of 16
+    (2, 257, 256, 3),      # the largest table, ragged tile
+    (1, 1, 1, 2),          # one token, one centroid
+    (2, 5000, 255, 2),
+    (2, 300, 64, 0),       # no iteration: the initial tokens
+])
+def test_fit_parity(H, N, C, iters):
+    """Lloyd k-means on the GPU equals the oracle's bit for bit: the tensor
+    cores only screen, every assignment is decided on the sequential fp32
+    distance and every mean is the fp32 rounding of the exact mean."""
+    _, k, _ = make_chunk(11 + N, N, H)
     kb = synth.bits(k)
     ref = orc.fit_centroids(kb, C, iters)
     cfg = qwm.config(H, C, kmeans_iters=iters)
-    got = qwm.qwm_fit_centroids(cfg, dev(k))
-    torch.cuda.synchronize()
-    g = synth.bits(got.cpu())
-    # same assignments against both tables, and the k-means objective agrees
-    exact = np.array_equal(g, ref["centroids"])
-    xf = orc.bf16_to_f32(kb).astype(np.float64)
-    for h in range(H):
-        cg = orc.bf16_to_f32(g[h]).astype(np.float64)
-        cr = orc.bf16_to_f32(ref["centroids"][h]).astype(np.float64)
-        dg = ((xf[:, h, None, :] - cg[None]) ** 2).sum(-1)
-        dr = ((xf[:, h, None, :] - cr[None]) ** 2).sum(-1)
-        agree = (dg.argmin(1) == dr.argmin(1)).mean()
-        assert agree >= 0.999 or exact
-        og, orf = dg.min(1).sum(), dr.min(1).sum()
-        assert abs(og - orf) <= 1e-4 * orf
-    # k = C = 1 iteration-free case: init tokens exactly
-    cfg0 = qwm.config(H, C, kmeans_iters=0)
-    got0 = synth.bits(qwm.qwm_fit_centroids(cfg0, dev(k)).cpu())
-    assert np.array_equal(got0, orc.fit_centroids(kb, C, 0)["centroids"])
+    got = synth.bits(qwm.qwm_fit_centroids(cfg, dev(k)).cpu())
+    nbad = int((got != ref["centroids"]).any(-1).sum())
+    assert nbad == 0, f"{nbad} of {H * C} centroids differ"
+
+
+def test_fit_parity_full_size_sampled():
+    """The Wan-14B-shaped Keys and Values (40 heads, 4680 tokens, 256
+    centroids, 10 iterations); the oracle runs on three sampled heads."""
+    wl = synth.WORKLOADS["wan14b_layer"]
+    src = synth.ChunkSource(wl)
+    _, k, v = src.chunk(0)
+    cfg = qwm.config(wl.heads, wl.centroids, kmeans_iters=wl.kmeans_iters)
+    heads = [0, 21, 39]
+    for x in (k, v):
+        got = synth.bits(qwm.qwm_fit_centroids(cfg, dev(x)).cpu())
+        ref = orc.fit_centroids(synth.bits(x[:, heads].contiguous()), wl.centroids, wl.kmeans_iters)
+        assert np.array_equal(got[heads], ref["centroids"])
 
 
 def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, window=0, max_chunks=None,

@@ -34,7 +34,7 @@ def test_noalloc_fit_matches_workspace_fit_on_consecutive_calls():
 def test_noalloc_fit_rejects_sizes_beyond_the_static_scratch():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
-    cfg = qwm.config(64, 256, kmeans_iters=1)  # 64*256*(12*128+4) bytes > 16 MiB
+    cfg = qwm.config(64, 256, kmeans_iters=1)  # centroids 8 MiB + operand images 8 MiB + more > 16 MiB
     x = synth.gaussian_bf16(3, 300, 64, 128).cuda()
     with pytest.raises(qwm.QwmError) as e:
         qwm.qwm_fit_centroids_noalloc(cfg, x)
