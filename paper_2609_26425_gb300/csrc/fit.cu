@@ -34,17 +34,22 @@ namespace {
 
 using namespace ptx;
 
-constexpr int AT = 128;                       // tokens per tile = threads per assign CTA
+constexpr int AT = 128;                       // tokens per tile
+constexpr int AEW = 8;                        // epilogue warps: rows 32 (w & 3) + lane, column half w >> 2
+constexpr int ANT = (AEW + 1) * 32;           // + one producer / MMA warp
 constexpr int kPairCap = 1024;                // (row, centroid) pairs rescored per tile
-constexpr int kRowCap = 8;                    // candidates listed per row
-constexpr int A_X = 0;                        // token tile: 2 x [128 rows][128 B] bf16
-constexpr int A_IMG = 32768;                  // operand images hi, lo: 2 x 2 x [Npad][128 B]
-constexpr int A_NRM = A_IMG + 131072;         // |mu_j|^2 [256]
-constexpr int A_PJ = A_NRM + 1024;            // pair (row << 16 | j) [kPairCap]
+constexpr int kRowCap = 8;                    // candidates per row
+constexpr int A_X = 0;                        // 2 token tiles, each 2 x [128 rows][128 B] bf16
+constexpr int A_IMG = 65536;                  // operand images hi, lo: 2 x 2 x [Npad][128 B]
+constexpr int A_NRM = A_IMG + 131072;         // |mu_j|^2 [256] for each TMEM buffer
+constexpr int A_PJ = A_NRM + 2048;            // pair (row << 16 | j) [kPairCap]
 constexpr int A_PD = A_PJ + kPairCap * 4;     // pair distance [kPairCap]
 constexpr int A_ROW = A_PD + kPairCap * 4;    // row: first slot << 16 | count (0xFFFF: full scan)
-constexpr int A_BAR = A_ROW + AT * 4;         // 3 mbarriers, pair counter, flag, TMEM slot
-constexpr int A_SMEM = A_BAR + 64 + 1024;
+constexpr int A_MIN = A_ROW + AT * 4;         // [2 halves][128] partial minima
+constexpr int A_CNT = A_MIN + 2 * AT * 4;     // [2 halves][128] candidate counts
+constexpr int A_CND = A_CNT + 2 * AT * 4;     // [128][2 halves][kRowCap] candidates (u8)
+constexpr int A_BAR = A_CND + AT * 2 * kRowCap;   // mbarriers, pair counter, flag, TMEM slot
+constexpr int A_SMEM = A_BAR + 128 + 1024;
 
 // Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in two
 // 128-byte-swizzled blocks of `rows` rows x 64 two-byte elements.
@@ -121,34 +126,44 @@ __global__ void __launch_bounds__(512) fit_prep(const FitArgs a) {
 }
 
 // Assignment of every token (see the file comment).  Units are (head, tile)
-// in head-major order, split into contiguous runs over the CTAs, so a CTA
-// loads the images of a head once per run.
-__global__ void __launch_bounds__(AT, 1)
+// in head-major order, split into contiguous runs over the CTAs.  Warp 8 loads
+// (TMA) and multiplies (tcgen05) tile t + 1 into the second token buffer and
+// TMEM accumulator while warps 0-7 finish tile t: two warps per row, one per
+// column half of the accumulator, meeting in shared memory.
+__global__ void __launch_bounds__(ANT, 1)
     fit_assign(const FitArgs a, const __grid_constant__ CUtensorMap tm, int tiles, int units) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  const int tid = threadIdx.x, warp = tid >> 5, row = tid;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int C = a.C, Npad = a.Npad;
-  uint8_t* sX = sm + A_X;
-  const float* sNrm = reinterpret_cast<const float*>(sm + A_NRM);
   uint32_t* sPJ = reinterpret_cast<uint32_t*>(sm + A_PJ);
   float* sPD = reinterpret_cast<float*>(sm + A_PD);
   uint32_t* sRow = reinterpret_cast<uint32_t*>(sm + A_ROW);
-  const uint32_t bar_tma = smem_u32(sm + A_BAR), bar_img = bar_tma + 8, bar_mma = bar_tma + 16;
-  int* s_np = reinterpret_cast<int*>(sm + A_BAR + 24);
-  volatile int* s_err = reinterpret_cast<volatile int*>(sm + A_BAR + 28);
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + A_BAR + 32);
+  float* sMin = reinterpret_cast<float*>(sm + A_MIN);
+  int* sCnt = reinterpret_cast<int*>(sm + A_CNT);
+  uint8_t* sCnd = sm + A_CND;
+  const uint32_t bars = smem_u32(sm + A_BAR);
+  auto bar_tma = [&](int b) { return bars + 8 * b; };          // token tile b landed
+  auto bar_mma = [&](int b) { return bars + 16 + 8 * b; };     // accumulator b complete
+  auto bar_free = [&](int b) { return bars + 32 + 8 * b; };    // tile b and accumulator b consumed
+  const uint32_t bar_img = bars + 48;
+  int* s_np = reinterpret_cast<int*>(sm + A_BAR + 64);
+  volatile int* s_err = reinterpret_cast<volatile int*>(sm + A_BAR + 68);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + A_BAR + 72);
   uint32_t ncols = 32;
   while ((int)ncols < Npad) ncols <<= 1;
 
   if (warp == 0) {
-    tmem_alloc(smem_u32(tslot), ncols);
+    tmem_alloc(smem_u32(tslot), 2 * ncols);
     tmem_relinquish();
   }
   if (tid == 0) {
-    mbar_init(bar_tma, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar_tma(b), 1);
+      mbar_init(bar_mma(b), 1);
+      mbar_init(bar_free(b), AEW);
+    }
     mbar_init(bar_img, 1);
-    mbar_init(bar_mma, 1);
     fence_mbar_init();
     *s_np = 0;
     *s_err = 0;
@@ -156,170 +171,191 @@ __global__ void __launch_bounds__(AT, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tD = *tslot;
-  const uint32_t lrow = (uint32_t)(warp * 32) << 16;
-  const int nchunk = (Npad + 31) >> 5;
-  const uint32_t id = idesc_f16(128, Npad, false, true);
-
+  const uint32_t tbase = *tslot;
   const int u0 = (int)((int64_t)blockIdx.x * units / gridDim.x);
   const int u1 = (int)((int64_t)(blockIdx.x + 1) * units / gridDim.x);
-  uint32_t ph_tma = 0, ph_img = 0, ph_mma = 0;
-  int cur_h = -1;
-  float nmx = 0.0f;
-  for (int u = u0; u < u1; ++u) {
-    const int h = u / tiles, tile = u - h * tiles;
-    if (h != cur_h) {  // this head's operand images and norms (earlier MMAs have completed)
-      if (tid == 0) {
-        const uint32_t ib = (uint32_t)Npad * 512u;
-        mbar_arrive_expect_tx(bar_img, ib + (uint32_t)Npad * 4u);
-        bulk_g2s(smem_u32(sm + A_IMG), a.img + (size_t)h * ib, ib, bar_img);
-        bulk_g2s(smem_u32(sm + A_NRM), a.nrm + (size_t)h * Npad, (uint32_t)Npad * 4u, bar_img);
-      }
-      if (!mbar_wait(bar_img, ph_img)) *s_err = 1;
-      ph_img ^= 1;
-      nmx = __uint_as_float(a.nmax[h]);
-      cur_h = h;
-    }
-    if (tid == 0) {
-      mbar_arrive_expect_tx(bar_tma, 32768);
-      tma_load_3d(smem_u32(sX), &tm, 0, h, tile * 128, bar_tma);
-      tma_load_3d(smem_u32(sX + 16384), &tm, 64, h, tile * 128, bar_tma);
-    }
-    if (!mbar_wait(bar_tma, ph_tma)) *s_err = 1;
-    ph_tma ^= 1;
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (*s_err) break;
-    if (tid == 0) {
-      const uint32_t aX = smem_u32(sX), aI = smem_u32(sm + A_IMG);
-#pragma unroll
-      for (int half = 0; half < 2; ++half)
-#pragma unroll
-        for (int kb = 0; kb < 2; ++kb)
-#pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            umma_ss(tD, desc_sw128(aX + kb * 16384 + ks * 32),
-                    desc_sw128(aI + half * Npad * 256 + kb * Npad * 128 + ks * 32), id, (half | kb | ks) != 0);
-      umma_commit(bar_mma);
-    }
-    // |x|^2 of this row while the MMAs run (any order: it only sizes E)
-    float kx = 0.0f;
-#pragma unroll 4
-    for (int ch = 0; ch < 16; ++ch) {
-      const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
-      const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const float x0 = __uint_as_float(xw[p] << 16), x1 = __uint_as_float(xw[p] & 0xFFFF0000u);
-        kx = fmaf(x0, x0, fmaf(x1, x1, kx));
-      }
-    }
-    bool ok = mbar_wait(bar_mma, ph_mma);
-    ph_mma ^= 1;
-    ok = __all_sync(0xFFFFFFFFu, ok);
-    tc_fence_after();
-    if (!ok) *s_err = 1;
+  const int T = u1 - u0;
 
-    // ---- smallest dt, then the candidates within 2E of it
-    float mn = INFINITY;
-    if (ok) {
+  if (warp == AEW) {
+    // ---------------- producer / MMA issuer
+    if (lane == 0) {
+      const uint32_t id = idesc_f16(128, Npad, false, true);
+      const uint32_t aI = smem_u32(sm + A_IMG);
+      const uint32_t ib = (uint32_t)Npad * 512u;
+      int cur_h = -1;
+      uint32_t ph_img = 0;
+      for (int t = 0; t < T; ++t) {
+        const int u = u0 + t, h = u / tiles, tile = u - h * tiles, b = t & 1;
+        if (t >= 2 && !mbar_wait(bar_free(b), ((t >> 1) - 1) & 1)) { *s_err = 1; break; }
+        if (h != cur_h) {
+          // the previous head's MMAs read the images: wait for them, then load this head's
+          if (t >= 1 && !mbar_wait(bar_mma((t - 1) & 1), ((t - 1) >> 1) & 1)) { *s_err = 1; break; }
+          mbar_arrive_expect_tx(bar_img, ib);
+          bulk_g2s(aI, a.img + (size_t)h * ib, ib, bar_img);
+          if (!mbar_wait(bar_img, ph_img)) { *s_err = 1; break; }
+          ph_img ^= 1;
+          cur_h = h;
+        }
+        const uint32_t aX = smem_u32(sm + A_X + b * 32768);
+        mbar_arrive_expect_tx(bar_tma(b), 32768u + (uint32_t)Npad * 4u);
+        tma_load_3d(aX, &tm, 0, h, tile * 128, bar_tma(b));
+        tma_load_3d(aX + 16384, &tm, 64, h, tile * 128, bar_tma(b));
+        bulk_g2s(smem_u32(sm + A_NRM + b * 1024), a.nrm + (size_t)h * Npad, (uint32_t)Npad * 4u, bar_tma(b));
+        if (!mbar_wait(bar_tma(b), (t >> 1) & 1)) { *s_err = 1; break; }
+        tc_fence_after();
+        const uint32_t tD = tbase + (uint32_t)b * ncols;
+#pragma unroll
+        for (int half = 0; half < 2; ++half)
+#pragma unroll
+          for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+              umma_ss(tD, desc_sw128(aX + kb * 16384 + ks * 32),
+                      desc_sw128(aI + half * Npad * 256 + kb * Npad * 128 + ks * 32), id, (half | kb | ks) != 0);
+        umma_commit(bar_mma(b));
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue: warps 0-7
+    const int hf = warp >> 2, row = (warp & 3) * 32 + lane;
+    const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
+    const int nchunk = (Npad + 31) >> 5;
+    const int ch0 = hf ? (nchunk + 1) >> 1 : 0, ch1 = hf ? nchunk : (nchunk + 1) >> 1;
+    for (int t = 0; t < T; ++t) {
+      const int u = u0 + t, h = u / tiles, tile = u - h * tiles, b = t & 1;
+      const uint8_t* sX = sm + A_X + b * 32768;
+      const float* sNrm = reinterpret_cast<const float*>(sm + A_NRM + b * 1024);
+      const uint32_t tD = tbase + (uint32_t)b * ncols;
+      bool ok = mbar_wait(bar_mma(b), (t >> 1) & 1);
+      ok = __all_sync(0xFFFFFFFFu, ok);
+      tc_fence_after();
+      if (!ok) *s_err = 1;
+      // |x|^2 of the row (any order: it only sizes E)
+      float kx = 0.0f;
+#pragma unroll 4
+      for (int ch = 0; ch < 16; ++ch) {
+        const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
+        const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const float x0 = __uint_as_float(xw[p] << 16), x1 = __uint_as_float(xw[p] & 0xFFFF0000u);
+          kx = fmaf(x0, x0, fmaf(x1, x1, kx));
+        }
+      }
+      // smallest dt of this half
+      float mn = INFINITY;
+      if (ok) {
 #pragma unroll 1
-      for (int cb = 0; cb < nchunk; ++cb) {
-        float v[32];
-        tmem_ld32(tD + lrow + cb * 32, v);
+        for (int cb = ch0; cb < ch1; ++cb) {
+          float v[32];
+          tmem_ld32(tD + lrow + cb * 32, v);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int j = cb * 32 + e;
-          const float dt = j < C ? fmaf(-2.0f, v[e], sNrm[j]) : INFINITY;
-          mn = fminf(mn, dt);
+          for (int e = 0; e < 32; ++e) {
+            const int j = cb * 32 + e;
+            mn = fminf(mn, j < C ? fmaf(-2.0f, v[e], sNrm[j]) : INFINITY);
+          }
         }
       }
-    }
-    const float thr = mn + 2.0f * ldexpf(kx + nmx, -11);
-    const int64_t n = (int64_t)tile * 128 + row;
-    const bool valid = n < a.N;
-    bool full = !(thr < INFINITY);
-    int cnt = 0;
-    int cj[kRowCap];
-#pragma unroll
-    for (int s2 = 0; s2 < kRowCap; ++s2) cj[s2] = 0;
-    if (ok) {
+      sMin[hf * AT + row] = mn;
+      named_bar_sync(1, AEW * 32);
+      mn = fminf(sMin[row], sMin[AT + row]);
+      const float thr = mn + 2.0f * ldexpf(kx + __uint_as_float(a.nmax[h]), -11);
+      // this half's candidates, ascending
+      int cnt = 0;
+      uint8_t* cand = sCnd + (row * 2 + hf) * kRowCap;
+      if (ok && thr < INFINITY) {
 #pragma unroll 1
-      for (int cb = 0; cb < nchunk; ++cb) {
-        float v[32];
-        tmem_ld32(tD + lrow + cb * 32, v);
+        for (int cb = ch0; cb < ch1; ++cb) {
+          float v[32];
+          tmem_ld32(tD + lrow + cb * 32, v);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int j = cb * 32 + e;
-          if (j < C && fmaf(-2.0f, v[e], sNrm[j]) <= thr) {
-#pragma unroll
-            for (int s2 = 0; s2 < kRowCap; ++s2)
-              if (s2 == cnt) cj[s2] = j;
-            ++cnt;
+          for (int e = 0; e < 32; ++e) {
+            const int j = cb * 32 + e;
+            if (j < C && fmaf(-2.0f, v[e], sNrm[j]) <= thr) {
+              if (cnt < kRowCap) cand[cnt] = (uint8_t)j;
+              ++cnt;
+            }
           }
         }
       }
-    }
-    full = full || cnt > kRowCap || cnt == 0;
-    uint32_t rinfo = 0;
-    if (valid && ok && !full && cnt > 1) {
-      const int base = atomicAdd(s_np, cnt);
-      if (base + cnt <= kPairCap) {
-#pragma unroll
-        for (int s2 = 0; s2 < kRowCap; ++s2)
-          if (s2 < cnt) sPJ[base + s2] = ((uint32_t)row << 16) | (uint32_t)cj[s2];
-        rinfo = ((uint32_t)base << 16) | (uint32_t)cnt;
-      } else {
-        full = true;
-      }
-    }
-    if (full) rinfo = 0xFFFFu;
-    sRow[row] = rinfo;
-    tc_fence_before();
-    __syncthreads();
-    // ---- exact rescoring of the listed pairs, spread over the CTA
-    const int np = min(*s_np, kPairCap);
-    const float* muh = a.cent + (size_t)cur_h * C * 128;
-    for (int p = tid; p < np; p += AT) {
-      const uint32_t pj = sPJ[p];
-      sPD[p] = exact_dist(sX, (int)(pj >> 16), muh + (size_t)(pj & 0xFFFFu) * 128);
-    }
-    __syncthreads();
-    if (valid && ok) {
-      int best = cj[0];
-      if (rinfo == 0xFFFFu) {  // every centroid, sequentially (non-finite rows, crowded bands)
-        float bd = 0.0f;
-        for (int j = 0; j < C; ++j) {
-          const float dj = exact_dist(sX, row, muh + (size_t)j * 128);
-          if (j == 0 || dj < bd) {
-            bd = dj;
-            best = j;
+      sCnt[hf * AT + row] = (ok && thr < INFINITY) ? cnt : -1;
+      tc_fence_before();
+      named_bar_sync(1, AEW * 32);
+      // the row owner (half 0) merges: one candidate decides, a few go to the pair list
+      const int64_t n = (int64_t)tile * 128 + row;
+      const bool valid = n < a.N;
+      int best = 0;
+      if (hf == 0) {
+        const int c0 = sCnt[row], c1 = sCnt[AT + row];
+        const int tot = c0 + c1;
+        uint32_t rinfo = 0;
+        if (c0 < 0 || c1 < 0 || tot == 0 || tot > kRowCap) {
+          rinfo = 0xFFFFu;  // every centroid, sequentially
+        } else if (tot == 1) {
+          best = c0 ? sCnd[row * 2 * kRowCap] : sCnd[(row * 2 + 1) * kRowCap];
+        } else if (valid) {
+          const int base = atomicAdd(s_np, tot);
+          if (base + tot <= kPairCap) {
+            for (int s2 = 0; s2 < tot; ++s2) {
+              const int j = s2 < c0 ? sCnd[row * 2 * kRowCap + s2] : sCnd[(row * 2 + 1) * kRowCap + s2 - c0];
+              sPJ[base + s2] = ((uint32_t)row << 16) | (uint32_t)j;
+            }
+            rinfo = ((uint32_t)base << 16) | (uint32_t)tot;
+          } else {
+            rinfo = 0xFFFFu;
           }
         }
-      } else if (rinfo != 0) {
-        const int base = (int)(rinfo >> 16), c2 = (int)(rinfo & 0xFFFFu);
-        float bd = sPD[base];
-        best = (int)(sPJ[base] & 0xFFFFu);
-        for (int s2 = 1; s2 < c2; ++s2)
-          if (sPD[base + s2] < bd) {  // ascending j: the lower index keeps a tie
-            bd = sPD[base + s2];
-            best = (int)(sPJ[base + s2] & 0xFFFFu);
-          }
+        sRow[row] = rinfo;
       }
-      a.asg[(size_t)cur_h * a.N + n] = (uint8_t)best;
-      atomicAdd(a.counts + (size_t)cur_h * C + best, 1);
+      named_bar_sync(1, AEW * 32);
+      // exact rescoring of the listed pairs, spread over the epilogue warps
+      const int np = min(*s_np, kPairCap);
+      const float* muh = a.cent + (size_t)h * C * 128;
+      for (int p = tid; p < np; p += AEW * 32) {
+        const uint32_t pj = sPJ[p];
+        sPD[p] = exact_dist(sX, (int)(pj >> 16), muh + (size_t)(pj & 0xFFFFu) * 128);
+      }
+      named_bar_sync(1, AEW * 32);
+      if (hf == 0 && valid && ok) {
+        const uint32_t rinfo = sRow[row];
+        if (rinfo == 0xFFFFu) {
+          float bd = 0.0f;
+          for (int j = 0; j < C; ++j) {
+            const float dj = exact_dist(sX, row, muh + (size_t)j * 128);
+            if (j == 0 || dj < bd) {
+              bd = dj;
+              best = j;
+            }
+          }
+        } else if (rinfo != 0) {
+          const int base = (int)(rinfo >> 16), c2 = (int)(rinfo & 0xFFFFu);
+          float bd = sPD[base];
+          best = (int)(sPJ[base] & 0xFFFFu);
+          for (int s2 = 1; s2 < c2; ++s2)
+            if (sPD[base + s2] < bd) {  // ascending j: the lower index keeps a tie
+              bd = sPD[base + s2];
+              best = (int)(sPJ[base + s2] & 0xFFFFu);
+            }
+        }
+        a.asg[(size_t)h * a.N + n] = (uint8_t)best;
+        atomicAdd(a.counts + (size_t)h * C + best, 1);
+      }
+      fence_proxy_async_smem();  // generic reads of tile b before the next copy into it
+      tc_fence_before();
+      // one vote, so that every epilogue warp leaves the loop together
+      const bool go = named_bar_and(1, AEW * 32, *s_err == 0);
+      if (tid == 0) *s_np = 0;
+      if (lane == 0) mbar_arrive(bar_free(b));
+      if (!go) break;
     }
-    fence_proxy_async_smem();  // generic reads of the tile before the next copy overwrites it
-    __syncthreads();
-    if (tid == 0) *s_np = 0;
   }
   if (tid == 0 && *s_err) atomicCAS(a.status, 0, (int)QWM_ERR_TIMEOUT);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tD, ncols);
+    tmem_dealloc(tbase, 2 * ncols);
   }
 }
 
@@ -354,9 +390,46 @@ __global__ void __launch_bounds__(1024) fit_scatter(const FitArgs a) {
   }
 }
 
+// Largest bf16 exponent field over each head's tokens: it fixes the unit
+// 2^U of the exact fixed-point member sums (U = emax - 134 - room).
+__global__ void __launch_bounds__(256) fit_scale(const FitArgs a) {
+  const int h = blockIdx.y, lane = threadIdx.x & 31;
+  uint32_t mx = 0;
+  for (int64_t n = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); n < a.N; n += (int64_t)gridDim.x * 8) {
+    const uint2 xv = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)n * a.H + h) * 128 + 4 * lane));
+    mx = max(mx, max(max((xv.x >> 7) & 0xFFu, (xv.x >> 23) & 0xFFu), max((xv.y >> 7) & 0xFFu, (xv.y >> 23) & 0xFFu)));
+  }
+  mx = __reduce_max_sync(0xFFFFFFFFu, mx);
+  if (lane == 0) atomicMax(a.emax + h, (int)mx);
+}
+
 // New centroid j of head h: the fp32 rounding of the fp64 member mean (kept
 // when the cluster is empty); then its images and norm.  One warp each, lane =
-// four channels; the member rows are read four at a time.
+// four channels, member rows read four at a time.
+//   The member sum is exact and independent of order.  A normal bf16 value is
+//   (128 + f) 2^(e - 134); with U = emax - 134 - room every member is the
+//   integer (128 + f) << (e - 134 - U) < 2^(8 + room) in units of 2^U, and N
+//   of them add in int64 without overflow.  A member outside that grid (tiny,
+//   subnormal, inf or NaN) sends the cluster to fp64 sums instead.
+//   The mean RN32(RN64(S / n)): q = S * RN64(1/n) lies within 2.5 ulp of
+//   RN64(S / n), so both round to the same fp32 value unless q is within a
+//   few ulp of a point halfway between two fp32 values; there (and outside the
+//   fp32 normal range) the exact fp64 division decides.
+__device__ __forceinline__ float mean_of(int64_t k, int U, double invs, double dc, bool& exact_ok) {
+  const double kd = (double)k;
+  if (!((double)(kd) == (double)k && (long long)kd == k)) {
+    exact_ok = false;
+    return 0.0f;
+  }
+  const double q = kd * invs;
+  const long long bits = __double_as_longlong(q);
+  const int ex = (int)((bits >> 52) & 0x7FF);
+  const long long lo = bits & ((1LL << 29) - 1);
+  const bool near = (lo > (1LL << 28) - 16 && lo < (1LL << 28) + 16) || ex < 1023 - 126 || ex > 1023 + 127;
+  if (k != 0 && near) return __double2float_rn(__ddiv_rn(ldexp(kd, U), dc));
+  return __double2float_rn(q);
+}
+
 __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
   const int lane = threadIdx.x & 31;
   const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -366,8 +439,21 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
   float4* cr = reinterpret_cast<float4*>(a.cent + (size_t)w * 128) + lane;
   float4 m;
   if (cnt > 0) {
-    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
     const int32_t* lst = a.list + (size_t)h * a.N + (base < a.N ? base : 0);
+    const int U = a.emax[h] - 134 - a.room;
+    int64_t k0 = 0, k1 = 0, k2 = 0, k3 = 0;
+    bool grid_ok = true;
+    auto fix = [&](uint32_t b16) -> int64_t {
+      const uint32_t e = (b16 >> 7) & 0xFFu, f = b16 & 0x7Fu;
+      if (e == 0) {
+        grid_ok = grid_ok && f == 0;
+        return 0;
+      }
+      const int sh = (int)e - 134 - U;
+      grid_ok = grid_ok && sh >= 0 && e != 255u;
+      const int64_t v = (int64_t)(128u + f) << (sh & 63);
+      return (b16 & 0x8000u) ? -v : v;
+    };
     for (int i = 0; i < cnt; i += 4) {
       uint2 xv[4];
 #pragma unroll
@@ -378,17 +464,36 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
           xv[k] = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)tok * a.H + h) * 128 + 4 * lane));
       }
 #pragma unroll
-      for (int k = 0; k < 4; ++k)
-        if (i + k < cnt) {
-          s0 += (double)__uint_as_float(xv[k].x << 16);
-          s1 += (double)__uint_as_float(xv[k].x & 0xFFFF0000u);
-          s2 += (double)__uint_as_float(xv[k].y << 16);
-          s3 += (double)__uint_as_float(xv[k].y & 0xFFFF0000u);
-        }
+      for (int k = 0; k < 4; ++k) {
+        k0 += fix(xv[k].x & 0xFFFFu);
+        k1 += fix(xv[k].x >> 16);
+        k2 += fix(xv[k].y & 0xFFFFu);
+        k3 += fix(xv[k].y >> 16);
+      }
     }
     const double dc = (double)cnt;
-    m = make_float4(__double2float_rn(__ddiv_rn(s0, dc)), __double2float_rn(__ddiv_rn(s1, dc)),
-                    __double2float_rn(__ddiv_rn(s2, dc)), __double2float_rn(__ddiv_rn(s3, dc)));
+    bool ok = __all_sync(0xFFFFFFFFu, grid_ok);
+    if (ok) {
+      const double invs = ldexp(__ddiv_rn(1.0, dc), U);
+      bool eo = true;
+      m = make_float4(mean_of(k0, U, invs, dc, eo), mean_of(k1, U, invs, dc, eo), mean_of(k2, U, invs, dc, eo),
+                      mean_of(k3, U, invs, dc, eo));
+      ok = __all_sync(0xFFFFFFFFu, eo);
+    }
+    if (!ok) {  // fp64 sums (exact for members of ordinary range)
+      double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+      for (int i = 0; i < cnt; ++i) {
+        const int64_t tok = lst[i];
+        if (tok < 0 || tok >= a.N) continue;
+        const uint2 xv = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)tok * a.H + h) * 128 + 4 * lane));
+        s0 += (double)__uint_as_float(xv.x << 16);
+        s1 += (double)__uint_as_float(xv.x & 0xFFFF0000u);
+        s2 += (double)__uint_as_float(xv.y << 16);
+        s3 += (double)__uint_as_float(xv.y & 0xFFFF0000u);
+      }
+      m = make_float4(__double2float_rn(__ddiv_rn(s0, dc)), __double2float_rn(__ddiv_rn(s1, dc)),
+                      __double2float_rn(__ddiv_rn(s2, dc)), __double2float_rn(__ddiv_rn(s3, dc)));
+    }
     *cr = m;
   } else {
     m = *cr;
@@ -424,7 +529,7 @@ size_t fit_workspace_bytes(int H, int d, int C, int64_t N) {
   b += (size_t)round_up((int64_t)H * C * d * 4, 256);           // cent
   b += (size_t)round_up((int64_t)H * Np * 512, 256);            // images
   b += (size_t)round_up((int64_t)H * Np * 4, 256);              // norms
-  b += (size_t)round_up((int64_t)H * 4, 256);                   // largest norm
+  b += 2 * (size_t)round_up((int64_t)H * 4, 256);               // largest norm, largest exponent
   b += 2 * (size_t)round_up((int64_t)H * C * 4, 256);           // counts, offsets
   b += (size_t)round_up((int64_t)H * N, 256);                   // assignment
   b += (size_t)round_up((int64_t)H * N * 4, 256);               // member lists
@@ -444,6 +549,11 @@ void fit_carve(FitArgs& a, uint8_t* ws) {
   a.img = take((int64_t)a.H * a.Npad * 512);
   a.nrm = reinterpret_cast<float*>(take((int64_t)a.H * a.Npad * 4));
   a.nmax = reinterpret_cast<uint32_t*>(take((int64_t)a.H * 4));
+  a.emax = reinterpret_cast<int32_t*>(take((int64_t)a.H * 4));
+  // member sums of at most N values below 2^(8 + room) each stay below 2^61
+  int lg = 0;
+  while (((int64_t)1 << lg) < a.N + 1) ++lg;
+  a.room = 53 - lg;
   a.counts = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.offs = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.asg = take((int64_t)a.H * a.N);
@@ -454,6 +564,7 @@ cudaError_t launch_fit(const FitArgs& a, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaMemsetAsync(a.status, 0, 4, st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(a.nmax, 0, (size_t)a.H * 4, st)) != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(a.emax, 0, (size_t)a.H * 4, st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(a.counts, 0, (size_t)a.H * a.C * 4, st)) != cudaSuccess) return e;
   const int64_t prep_warps = (int64_t)a.H * a.Npad;
   fit_prep<<<(unsigned)((prep_warps + 15) / 16), 512, 0, st>>>(a);
@@ -466,8 +577,10 @@ cudaError_t launch_fit(const FitArgs& a, cudaStream_t st) {
     const int units = a.H * tiles;
     const int grid = units < sm_count() ? units : sm_count();
     const int64_t mean_warps = (int64_t)a.H * a.C;
+    const int64_t sb = (a.N + 7) / 8;
+    fit_scale<<<dim3((unsigned)(sb < 64 ? sb : 64), (unsigned)a.H), 256, 0, st>>>(a);
     for (int it = 0; it < a.iters; ++it) {
-      fit_assign<<<grid, AT, A_SMEM, st>>>(a, tm, tiles, units);
+      fit_assign<<<grid, ANT, A_SMEM, st>>>(a, tm, tiles, units);
       fit_scatter<<<a.H, 1024, 0, st>>>(a);
       fit_means<<<(unsigned)((mean_warps + 15) / 16), 512, 0, st>>>(a);
     }

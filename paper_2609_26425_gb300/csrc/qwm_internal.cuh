@@ -136,6 +136,8 @@ struct FitArgs {
   uint8_t* img;                // [H][2][Npad * 256] bf16 MMA operand images: hi, lo
   float* nrm;                  // [H][Npad] squared centroid norms
   uint32_t* nmax;              // [H] largest squared norm (fp32 bits)
+  int32_t* emax;               // [H] largest bf16 exponent field of the head's tokens
+  int room;                    // fixed-point headroom bits of the exact member sums
   int32_t* counts;             // [H][C] members per cluster
   int32_t* offs;               // [H][C] first member slot
   uint8_t* asg;                // [H][N] assignment
