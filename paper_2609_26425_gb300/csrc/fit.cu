@@ -35,7 +35,7 @@ namespace {
 using namespace ptx;
 
 constexpr int AT = 128;                       // tokens per tile
-constexpr int AEW = 8;                        // epilogue warps: rows 32 (w & 3) + lane, column half w >> 2
+constexpr int AEW = 16;                       // epilogue warps: rows 32 (w & 3) + lane, column quarter w >> 2
 constexpr int ANT = (AEW + 1) * 32;           // + one producer / MMA warp
 constexpr int kPairCap = 1024;                // (row, centroid) pairs rescored per tile
 constexpr int kRowCap = 8;                    // candidates per row
@@ -45,10 +45,10 @@ constexpr int A_NRM = A_IMG + 131072;         // |mu_j|^2 [256] for each TMEM bu
 constexpr int A_PJ = A_NRM + 2048;            // pair (row << 16 | j) [kPairCap]
 constexpr int A_PD = A_PJ + kPairCap * 4;     // pair distance [kPairCap]
 constexpr int A_ROW = A_PD + kPairCap * 4;    // row: first slot << 16 | count (0xFFFF: full scan)
-constexpr int A_MIN = A_ROW + AT * 4;         // [2 halves][128] partial minima
-constexpr int A_CNT = A_MIN + 2 * AT * 4;     // [2 halves][128] candidate counts
-constexpr int A_CND = A_CNT + 2 * AT * 4;     // [128][2 halves][kRowCap] candidates (u8)
-constexpr int A_BAR = A_CND + AT * 2 * kRowCap;   // mbarriers, pair counter, flag, TMEM slot
+constexpr int A_MIN = A_ROW + AT * 4;         // [4 quarters][128] partial minima
+constexpr int A_CNT = A_MIN + 4 * AT * 4;     // [4 quarters][128] candidate counts
+constexpr int A_CND = A_CNT + 4 * AT * 4;     // [128][4 quarters][kRowCap] candidates (u8)
+constexpr int A_BAR = A_CND + AT * 4 * kRowCap;   // mbarriers, pair counter, flag, TMEM slot
 constexpr int A_SMEM = A_BAR + 128 + 1024;
 
 // Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in two
@@ -58,16 +58,19 @@ __device__ __forceinline__ int sw_off(int rows, int row, int ch) {
 }
 
 // The sequential fp32 distance of the definition: channel order, the
-// difference, its square and the running sum each rounded on its own.
+// difference, its square and the running sum each rounded on its own.  The
+// centroid row is fetched whole first (one memory round trip), then summed.
 __device__ float exact_dist(const uint8_t* sX, int row, const float* mu) {
+  float4 mv[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) mv[i] = __ldg(reinterpret_cast<const float4*>(mu) + i);
   float acc = 0.0f;
-#pragma unroll 2
+#pragma unroll
   for (int ch = 0; ch < 16; ++ch) {
     const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
-    const float4 m0 = __ldg(reinterpret_cast<const float4*>(mu + ch * 8));
-    const float4 m1 = __ldg(reinterpret_cast<const float4*>(mu + ch * 8 + 4));
     const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-    const float ms[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+    const float ms[8] = {mv[2 * ch].x, mv[2 * ch].y, mv[2 * ch].z, mv[2 * ch].w,
+                         mv[2 * ch + 1].x, mv[2 * ch + 1].y, mv[2 * ch + 1].z, mv[2 * ch + 1].w};
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
       const float xe = (e & 1) ? __uint_as_float(xw[e >> 1] & 0xFFFF0000u) : __uint_as_float(xw[e >> 1] << 16);
@@ -114,7 +117,7 @@ __global__ void __launch_bounds__(512) fit_prep(const FitArgs a) {
     uint8_t* hi = a.img + (size_t)h * 2 * a.Npad * 256;
     *reinterpret_cast<uint2*>(hi + off) = make_uint2(0, 0);
     *reinterpret_cast<uint2*>(hi + (size_t)a.Npad * 256 + off) = make_uint2(0, 0);
-    if (lane == 0) a.nrm[(size_t)h * a.Npad + j] = 0.0f;
+    if (lane == 0) a.nrm[(size_t)h * a.Npad + j] = INFINITY;  // padding columns never win
     return;
   }
   const int64_t src = ((int64_t)j * a.N) / a.C;
@@ -157,6 +160,10 @@ __global__ void __launch_bounds__(ANT, 1)
     tmem_alloc(smem_u32(tslot), 2 * ncols);
     tmem_relinquish();
   }
+  // norms past Npad are never copied in: +inf, so that columns beyond the
+  // MMA width (read when Npad is not a multiple of 32) never win
+  for (int i = tid; i < 512; i += ANT)
+    if ((i & 255) >= Npad) reinterpret_cast<float*>(sm + A_NRM)[i] = INFINITY;
   if (tid == 0) {
     for (int b = 0; b < 2; ++b) {
       mbar_init(bar_tma(b), 1);
@@ -217,90 +224,98 @@ __global__ void __launch_bounds__(ANT, 1)
     }
     __syncwarp();
   } else {
-    // ---------------- epilogue: warps 0-7
-    const int hf = warp >> 2, row = (warp & 3) * 32 + lane;
+    // ---------------- epilogue: warps 0-15
+    const int qt = warp >> 2, row = (warp & 3) * 32 + lane;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
     const int nchunk = (Npad + 31) >> 5;
-    const int ch0 = hf ? (nchunk + 1) >> 1 : 0, ch1 = hf ? nchunk : (nchunk + 1) >> 1;
+    const int ch0 = (qt * nchunk) >> 2, ch1 = ((qt + 1) * nchunk) >> 2;   // this quarter's 32-column chunks
     for (int t = 0; t < T; ++t) {
       const int u = u0 + t, h = u / tiles, tile = u - h * tiles, b = t & 1;
       const uint8_t* sX = sm + A_X + b * 32768;
-      const float* sNrm = reinterpret_cast<const float*>(sm + A_NRM + b * 1024);
+      const float4* sNrm4 = reinterpret_cast<const float4*>(sm + A_NRM + b * 1024);  // +inf past C
       const uint32_t tD = tbase + (uint32_t)b * ncols;
+      const int64_t n = (int64_t)tile * 128 + row;
+      const bool valid = n < a.N;
+      const float kx = valid ? a.xn2[(size_t)h * a.N + n] : 0.0f;
       bool ok = mbar_wait(bar_mma(b), (t >> 1) & 1);
       ok = __all_sync(0xFFFFFFFFu, ok);
       tc_fence_after();
       if (!ok) *s_err = 1;
-      // |x|^2 of the row (any order: it only sizes E)
-      float kx = 0.0f;
-#pragma unroll 4
-      for (int ch = 0; ch < 16; ++ch) {
-        const uint4 xv = *reinterpret_cast<const uint4*>(sX + sw_off(128, row, ch));
-        const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const float x0 = __uint_as_float(xw[p] << 16), x1 = __uint_as_float(xw[p] & 0xFFFF0000u);
-          kx = fmaf(x0, x0, fmaf(x1, x1, kx));
-        }
-      }
-      // smallest dt of this half
+      // smallest dt of this quarter
       float mn = INFINITY;
       if (ok) {
 #pragma unroll 1
-        for (int cb = ch0; cb < ch1; ++cb) {
-          float v[32];
-          tmem_ld32(tD + lrow + cb * 32, v);
+        for (int cb = ch0; cb < ch1; cb += 2) {
+          float v[64];
+          const int cb2 = cb + 1 < ch1 ? cb + 1 : cb;  // a lone last chunk is read twice (harmless for a minimum)
+          tmem_ld32x2(tD + lrow + cb * 32, tD + lrow + cb2 * 32, *reinterpret_cast<float(*)[32]>(v),
+                      *reinterpret_cast<float(*)[32]>(v + 32));
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int j = cb * 32 + e;
-            mn = fminf(mn, j < C ? fmaf(-2.0f, v[e], sNrm[j]) : INFINITY);
+          for (int e4 = 0; e4 < 16; ++e4) {
+            const float4 nr = sNrm4[(e4 < 8 ? cb : cb2) * 8 + (e4 & 7)];
+            mn = fminf(mn, fminf(fminf(fmaf(-2.0f, v[4 * e4], nr.x), fmaf(-2.0f, v[4 * e4 + 1], nr.y)),
+                                 fminf(fmaf(-2.0f, v[4 * e4 + 2], nr.z), fmaf(-2.0f, v[4 * e4 + 3], nr.w))));
           }
         }
       }
-      sMin[hf * AT + row] = mn;
+      sMin[qt * AT + row] = mn;
       named_bar_sync(1, AEW * 32);
-      mn = fminf(sMin[row], sMin[AT + row]);
+      mn = fminf(fminf(sMin[row], sMin[AT + row]), fminf(sMin[2 * AT + row], sMin[3 * AT + row]));
       const float thr = mn + 2.0f * ldexpf(kx + __uint_as_float(a.nmax[h]), -11);
-      // this half's candidates, ascending
+      // this quarter's candidates, ascending
       int cnt = 0;
-      uint8_t* cand = sCnd + (row * 2 + hf) * kRowCap;
+      uint8_t* cand = sCnd + (row * 4 + qt) * kRowCap;
       if (ok && thr < INFINITY) {
 #pragma unroll 1
-        for (int cb = ch0; cb < ch1; ++cb) {
-          float v[32];
-          tmem_ld32(tD + lrow + cb * 32, v);
+        for (int cb = ch0; cb < ch1; cb += 2) {
+          float v[64];
+          const int cb2 = cb + 1 < ch1 ? cb + 1 : cb;
+          tmem_ld32x2(tD + lrow + cb * 32, tD + lrow + cb2 * 32, *reinterpret_cast<float(*)[32]>(v),
+                      *reinterpret_cast<float(*)[32]>(v + 32));
+          const int ne = cb2 > cb ? 64 : 32;
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int j = cb * 32 + e;
-            if (j < C && fmaf(-2.0f, v[e], sNrm[j]) <= thr) {
-              if (cnt < kRowCap) cand[cnt] = (uint8_t)j;
-              ++cnt;
-            }
+          for (int e4 = 0; e4 < 16; ++e4) {
+            const float4 nr = sNrm4[(e4 < 8 ? cb : cb2) * 8 + (e4 & 7)];
+            const float d4[4] = {fmaf(-2.0f, v[4 * e4], nr.x), fmaf(-2.0f, v[4 * e4 + 1], nr.y),
+                                 fmaf(-2.0f, v[4 * e4 + 2], nr.z), fmaf(-2.0f, v[4 * e4 + 3], nr.w)};
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (4 * e4 + q < ne && d4[q] <= thr) {
+                if (cnt < kRowCap) cand[cnt] = (uint8_t)(cb * 32 + 4 * e4 + q);
+                ++cnt;
+              }
           }
         }
       }
-      sCnt[hf * AT + row] = (ok && thr < INFINITY) ? cnt : -1;
+      sCnt[qt * AT + row] = (ok && thr < INFINITY) ? cnt : -1;
       tc_fence_before();
       named_bar_sync(1, AEW * 32);
-      // the row owner (half 0) merges: one candidate decides, a few go to the pair list
-      const int64_t n = (int64_t)tile * 128 + row;
-      const bool valid = n < a.N;
+      // the row owner (quarter 0) merges: one candidate decides, a few go to the pair list
       int best = 0;
-      if (hf == 0) {
-        const int c0 = sCnt[row], c1 = sCnt[AT + row];
-        const int tot = c0 + c1;
+      if (qt == 0) {
+        int c[4], tot = 0;
+        bool bad = false;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          c[q] = sCnt[q * AT + row];
+          bad = bad || c[q] < 0;
+          tot += c[q];
+        }
         uint32_t rinfo = 0;
-        if (c0 < 0 || c1 < 0 || tot == 0 || tot > kRowCap) {
+        if (bad || tot == 0 || tot > kRowCap) {
           rinfo = 0xFFFFu;  // every centroid, sequentially
         } else if (tot == 1) {
-          best = c0 ? sCnd[row * 2 * kRowCap] : sCnd[(row * 2 + 1) * kRowCap];
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (c[q]) best = sCnd[(row * 4 + q) * kRowCap];
         } else if (valid) {
           const int base = atomicAdd(s_np, tot);
           if (base + tot <= kPairCap) {
-            for (int s2 = 0; s2 < tot; ++s2) {
-              const int j = s2 < c0 ? sCnd[row * 2 * kRowCap + s2] : sCnd[(row * 2 + 1) * kRowCap + s2 - c0];
-              sPJ[base + s2] = ((uint32_t)row << 16) | (uint32_t)j;
-            }
+            int s2 = 0;
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              for (int k = 0; k < c[q]; ++k)
+                sPJ[base + s2++] = ((uint32_t)row << 16) | (uint32_t)sCnd[(row * 4 + q) * kRowCap + k];
             rinfo = ((uint32_t)base << 16) | (uint32_t)tot;
           } else {
             rinfo = 0xFFFFu;
@@ -316,8 +331,8 @@ __global__ void __launch_bounds__(ANT, 1)
         const uint32_t pj = sPJ[p];
         sPD[p] = exact_dist(sX, (int)(pj >> 16), muh + (size_t)(pj & 0xFFFFu) * 128);
       }
-      named_bar_sync(1, AEW * 32);
-      if (hf == 0 && valid && ok) {
+      if (np > 0) named_bar_sync(1, AEW * 32);   // np is the same for every thread
+      if (qt == 0 && valid && ok) {
         const uint32_t rinfo = sRow[row];
         if (rinfo == 0xFFFFu) {
           float bd = 0.0f;
@@ -362,15 +377,26 @@ __global__ void __launch_bounds__(ANT, 1)
 // Counting sort of one head's tokens by cluster: offsets from the counts,
 // then each token to a slot of its cluster (any order within a cluster).
 __global__ void __launch_bounds__(1024) fit_scatter(const FitArgs a) {
-  __shared__ int s_off[256], s_cur[256];
-  const int h = blockIdx.x, tid = threadIdx.x, C = a.C;
-  if (tid == 0) {
-    int o = 0;
-    for (int j = 0; j < C; ++j) {
-      s_off[j] = o;
-      o += a.counts[(size_t)h * C + j];
+  __shared__ int s_off[256], s_cur[256], s_wsum[8];
+  const int h = blockIdx.x, tid = threadIdx.x, C = a.C, lane = tid & 31;
+  // exclusive prefix of the counts over j (warp scans, then the warp totals)
+  int v = 0, incl = 0;
+  if (tid < 256) {
+    v = tid < C ? a.counts[(size_t)h * C + tid] : 0;
+    incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += y;
     }
-    a.nmax[h] = 0u;  // rebuilt by fit_means
+    if (lane == 31) s_wsum[tid >> 5] = incl;
+  }
+  if (tid == 0) a.nmax[h] = 0u;  // rebuilt by fit_means
+  __syncthreads();
+  if (tid < 256) {
+    int wp = 0;
+    for (int k = 0; k < (tid >> 5); ++k) wp += s_wsum[k];
+    s_off[tid] = wp + incl - v;
   }
   __syncthreads();
   if (tid < C) {
@@ -390,14 +416,21 @@ __global__ void __launch_bounds__(1024) fit_scatter(const FitArgs a) {
   }
 }
 
-// Largest bf16 exponent field over each head's tokens: it fixes the unit
-// 2^U of the exact fixed-point member sums (U = emax - 134 - room).
+// Largest bf16 exponent field over each head's tokens, which fixes the unit
+// 2^U of the exact fixed-point member sums (U = emax - 134 - room), and |x|^2
+// of every token, which sizes the screening bound.
 __global__ void __launch_bounds__(256) fit_scale(const FitArgs a) {
   const int h = blockIdx.y, lane = threadIdx.x & 31;
   uint32_t mx = 0;
   for (int64_t n = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); n < a.N; n += (int64_t)gridDim.x * 8) {
     const uint2 xv = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)n * a.H + h) * 128 + 4 * lane));
     mx = max(mx, max(max((xv.x >> 7) & 0xFFu, (xv.x >> 23) & 0xFFu), max((xv.y >> 7) & 0xFFu, (xv.y >> 23) & 0xFFu)));
+    const float x0 = __uint_as_float(xv.x << 16), x1 = __uint_as_float(xv.x & 0xFFFF0000u);
+    const float x2 = __uint_as_float(xv.y << 16), x3 = __uint_as_float(xv.y & 0xFFFF0000u);
+    float n2 = fmaf(x0, x0, fmaf(x1, x1, fmaf(x2, x2, x3 * x3)));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) n2 += __shfl_xor_sync(0xFFFFFFFFu, n2, o);
+    if (lane == 0) a.xn2[(size_t)h * a.N + n] = n2;
   }
   mx = __reduce_max_sync(0xFFFFFFFFu, mx);
   if (lane == 0) atomicMax(a.emax + h, (int)mx);
@@ -532,6 +565,7 @@ size_t fit_workspace_bytes(int H, int d, int C, int64_t N) {
   b += 2 * (size_t)round_up((int64_t)H * 4, 256);               // largest norm, largest exponent
   b += 2 * (size_t)round_up((int64_t)H * C * 4, 256);           // counts, offsets
   b += (size_t)round_up((int64_t)H * N, 256);                   // assignment
+  b += (size_t)round_up((int64_t)H * N * 4, 256);               // token norms
   b += (size_t)round_up((int64_t)H * N * 4, 256);               // member lists
   return b;
 }
@@ -557,6 +591,7 @@ void fit_carve(FitArgs& a, uint8_t* ws) {
   a.counts = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.offs = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.asg = take((int64_t)a.H * a.N);
+  a.xn2 = reinterpret_cast<float*>(take((int64_t)a.H * a.N * 4));
   a.list = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.N * 4));
 }
 

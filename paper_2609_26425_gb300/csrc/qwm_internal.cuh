@@ -137,6 +137,7 @@ struct FitArgs {
   float* nrm;                  // [H][Npad] squared centroid norms
   uint32_t* nmax;              // [H] largest squared norm (fp32 bits)
   int32_t* emax;               // [H] largest bf16 exponent field of the head's tokens
+  float* xn2;                  // [H][N] |x|^2 of every token (fp32, any order)
   int room;                    // fixed-point headroom bits of the exact member sums
   int32_t* counts;             // [H][C] members per cluster
   int32_t* offs;               // [H][C] first member slot
