@@ -476,10 +476,12 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
     const int U = a.emax[h] - 134 - a.room;
     int64_t k0 = 0, k1 = 0, k2 = 0, k3 = 0;
     bool grid_ok = true;
+    // a member value in units of 2^U: (128 + f) << (e - 134 - U), below
+    // 2^(8 + room); zero stays zero; a value off the grid clears grid_ok
     auto fix = [&](uint32_t b16) -> int64_t {
       const uint32_t e = (b16 >> 7) & 0xFFu, f = b16 & 0x7Fu;
-      if (e == 0) {
-        grid_ok = grid_ok && f == 0;
+      if (e == 0u) {
+        grid_ok = grid_ok && f == 0u;
         return 0;
       }
       const int sh = (int)e - 134 - U;
@@ -487,21 +489,25 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
       const int64_t v = (int64_t)(128u + f) << (sh & 63);
       return (b16 & 0x8000u) ? -v : v;
     };
-    for (int i = 0; i < cnt; i += 4) {
-      uint2 xv[4];
+    for (int i0 = 0; i0 < cnt; i0 += 32) {
+      const int nb = min(32, cnt - i0);
+      const int my = lane < nb ? lst[i0 + lane] : -1;  // 32 member indices in one read
+      for (int kb = 0; kb < nb; kb += 8) {
+        uint2 xv[8];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        xv[k] = make_uint2(0, 0);
-        const int64_t tok = i + k < cnt ? (int64_t)lst[i + k] : -1;
-        if (tok >= 0 && tok < a.N)  // always, unless a timed-out assignment left stale lists
-          xv[k] = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)tok * a.H + h) * 128 + 4 * lane));
-      }
+        for (int k = 0; k < 8; ++k) {
+          const int tok = __shfl_sync(0xFFFFFFFFu, my, (kb + k) & 31);
+          xv[k] = make_uint2(0, 0);
+          if (kb + k < nb && tok >= 0 && tok < a.N)  // always, unless a timed-out assignment left stale lists
+            xv[k] = __ldg(reinterpret_cast<const uint2*>(a.x + ((size_t)tok * a.H + h) * 128 + 4 * lane));
+        }
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        k0 += fix(xv[k].x & 0xFFFFu);
-        k1 += fix(xv[k].x >> 16);
-        k2 += fix(xv[k].y & 0xFFFFu);
-        k3 += fix(xv[k].y >> 16);
+        for (int k = 0; k < 8; ++k) {
+          k0 += fix(xv[k].x & 0xFFFFu);
+          k1 += fix(xv[k].x >> 16);
+          k2 += fix(xv[k].y & 0xFFFFu);
+          k3 += fix(xv[k].y >> 16);
+        }
       }
     }
     const double dc = (double)cnt;

@@ -127,6 +127,22 @@ def test_fit_parity(H, N, C, iters):
     assert nbad == 0, f"{nbad} of {H * C} centroids differ"
 
 
+def test_fit_parity_off_grid_members():
+    """Entries of +-2^-45 among N(0, 1) values fall below the fixed-point grid
+    of the exact member sums (its unit is 2^-43 here), so their clusters take
+    the fp64 path; the fp64 sums stay exact (49 bits), and the fit must still
+    equal the oracle bit for bit."""
+    H, N, C, iters = 2, 300, 16, 3
+    g = torch.Generator().manual_seed(5)
+    x = torch.randn(N, H, 128, generator=g)
+    tiny = torch.rand(N, H, 128, generator=g) < 0.01
+    x = torch.where(tiny, torch.sign(x) * 2.0 ** -45, x).to(torch.bfloat16)
+    xb = synth.bits(x)
+    ref = orc.fit_centroids(xb, C, iters)
+    got = synth.bits(qwm.qwm_fit_centroids(qwm.config(H, C, kmeans_iters=iters), dev(x)).cpu())
+    assert np.array_equal(got, ref["centroids"])
+
+
 def test_fit_parity_full_size_sampled():
     """The Wan-14B-shaped Keys and Values (40 heads, 4680 tokens, 256
     centroids, 10 iterations); the oracle runs on three sampled heads."""
