@@ -254,3 +254,32 @@ def query_stats(q_bits, r: int):
     lam = lam[:, ::-1]
     vec = vec[:, :, ::-1]
     return M, w, np.ascontiguousarray(vec[:, :, :r]), np.ascontiguousarray(lam)
+
+
+# ---------------------------------------------------------------- token selection
+def top1(q_bits, k):
+    """Top-1 key of every query (Sec. 5, the top-1 token-selection shift
+    table): the key with the largest logit q . k, the first on ties (fp64,
+    numpy).  q_bits uint16 [Nq][H][d] (bf16 bits); k float64 [Nk][H][d].
+    Returns (idx int64 [H][Nq], margin [H][Nq]: best minus second-best logit
+    (inf with one key), scale [H][Nq]: |q| max_j |k_j|, which bounds every
+    logit)."""
+    q = bf16_to_f32(q_bits).astype(np.float64)
+    k = np.asarray(k, np.float64)
+    Nq, H, d = q.shape
+    idx = np.zeros((H, Nq), np.int64)
+    margin = np.full((H, Nq), np.inf)
+    scale = np.zeros((H, Nq))
+    for h in range(H):
+        L = q[:, h] @ k[:, h].T                      # [Nq][Nk]
+        idx[h] = np.argmax(L, axis=1)                # first maximum
+        if L.shape[1] > 1:
+            top2 = -np.partition(-L, 1, axis=1)[:, :2]
+            margin[h] = top2[:, 0] - top2[:, 1]
+        scale[h] = np.linalg.norm(q[:, h], axis=1) * np.linalg.norm(k[:, h], axis=1).max()
+    return idx, margin, scale
+
+
+def top1_shift(idx_ref, idx):
+    """Share of (query, head) pairs whose top-1 key differs from the reference's."""
+    return float(np.mean(np.asarray(idx_ref) != np.asarray(idx)))

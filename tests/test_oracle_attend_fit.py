@@ -166,3 +166,46 @@ def test_query_stats_cold_start_and_zero_queries(orc):
     assert np.all(w == 1.0) and np.all(U == 0.0) and np.all(M == 0.0)
     M, w, U, lam = orc.query_stats(np.zeros((5, H, d), np.uint16), r)
     assert np.all(w == 1.0) and np.all(lam == 0.0)
+
+
+# ------------------------------------------------------------------ token selection (top-1 key)
+def test_top1_brute_force_and_ties(orc):
+    """Pure-Python loops on a small case; a duplicated best key goes to the
+    lower index; a single key has margin inf."""
+    rng = np.random.default_rng(21)
+    Nq, Nk, H, d = 6, 9, 2, 128
+    qb = synth.bits(torch.from_numpy(rng.standard_normal((Nq, H, d)).astype(np.float32)).to(torch.bfloat16))
+    k = rng.standard_normal((Nk, H, d))
+    k[7] = k[2]                                   # a duplicate of key 2
+    idx, margin, _ = orc.top1(qb, k)
+    qf = orc.bf16_to_f32(qb).astype(np.float64)
+    for h in range(H):
+        for n in range(Nq):
+            logits = [sum(qf[n, h, c] * k[j, h, c] for c in range(d)) for j in range(Nk)]
+            best = max(logits)
+            first = min(j for j in range(Nk) if logits[j] == best)
+            assert idx[h, n] == first
+            assert idx[h, n] != 7                 # the duplicate never wins over key 2
+            srt = sorted(logits, reverse=True)
+            assert abs(margin[h, n] - (srt[0] - srt[1])) <= 1e-9 * abs(srt[0])
+    idx1, m1, _ = orc.top1(qb, k[:1])
+    assert np.all(idx1 == 0) and np.all(np.isinf(m1))
+
+
+def test_top1_closed_form_and_shift_ratio(orc):
+    """Keys along the unit channels with weights 1..d: query e_c picks the key
+    of channel c; swapping two keys changes exactly the queries that picked
+    them, so the shift ratio is 2/d."""
+    d = 128
+    k = np.zeros((d, 1, d))
+    k[np.arange(d), 0, np.arange(d)] = 1.0 + np.arange(d)
+    q = np.zeros((d, 1, d), np.float32)
+    q[np.arange(d), 0, np.arange(d)] = 1.0
+    qb = synth.bits(torch.from_numpy(q).to(torch.bfloat16))
+    idx, _, _ = orc.top1(qb, k)
+    assert np.array_equal(idx[0], np.arange(d))
+    k2 = k.copy()
+    k2[[3, 40]] = k2[[40, 3]]
+    idx2, _, _ = orc.top1(qb, k2)
+    assert orc.top1_shift(idx, idx) == 0.0
+    assert orc.top1_shift(idx, idx2) == 2.0 / d
