@@ -182,13 +182,16 @@ def run_gpu(args, wl, rank, world):
 
     # history: past_chunks appended through the product path (centroids fitted on the GPU)
     hist = qwm.Cache(cfg, N, wl.past_chunks, device=dev)
+    past = []
     for t in range(wl.past_chunks):
         _, k, v, w, U = chunk_inputs(t)
         kd, vd = k.to(dev), v.to(dev)
         kc = qwm.qwm_fit_centroids(cfg, kd, workspace=ws)
         vc = qwm.qwm_fit_centroids(cfg, vd, workspace=ws)
-        qwm.qwm_quantize_append(cfg, hist, kd, vd, kc, vc, w=None if w is None else w.to(dev),
-                                U=None if U is None else U.to(dev))
+        wd_t = None if w is None else w.to(dev)
+        Ud_t = None if U is None else U.to(dev)
+        qwm.qwm_quantize_append(cfg, hist, kd, vd, kc, vc, w=wd_t, U=Ud_t)
+        past.append((kd, vd, kc, vc, wd_t, Ud_t))
     # the new chunk
     q, k, v, w, U = chunk_inputs(wl.past_chunks)
     qd, kd, vd = q.to(dev), k.to(dev), v.to(dev)
@@ -304,6 +307,8 @@ def run_gpu(args, wl, rank, world):
     e_ms = job_time_ms(e_ms, world, dev)
 
     qs = query_stats_timing(qwm, cfg, qd, dev, max(3, min(args.steps, 20)), stream)
+    shift = top1_shift_measure(qwm, wl, hist, past, qd, dev)
+    del past
     fit_ms = fit_timing(qwm, cfg, kd, vd, ws, dev, max(3, min(args.steps, 10)), stream)
 
     pk = peaks()
@@ -342,11 +347,48 @@ def run_gpu(args, wl, rank, world):
                         "update_algorithmic_bytes": qs["update_bytes"],
                         "basis_ms": round(qs["basis_ms"], 4), "jacobi_sweeps": qs["sweeps"],
                         "l2": "update: 4 rotating copies of q (192 MB); basis: 256 MB flush before each launch"},
+        # quality: share of queries whose highest-logit cached key moves away from the bf16 keys' one
+        "top1_shift": shift,
         # chunk boundary, not on the step: Lloyd k-means tables of the chunk's Keys and Values
         "fit": {"ms_keys_and_values": round(fit_ms, 3), "kmeans_iters": wl.kmeans_iters,
                 "l2": "256 MB flush before each timed pair"},
     }
     return res
+
+
+def top1_shift_measure(qwm, wl, hist, past, qd, dev, every=9):
+    """Token-selection shift on the layer: the new chunk's queries (every 9th)
+    against the cached keys reconstructed from three caches of the same past
+    chunks: QVG (w = 1, nearest centroid, no PSAC), QSAC (w, top-M) and the
+    bench's own QSAC + PSAC cache; the reference is the bf16 keys."""
+    import torch
+    H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
+    qs = qd[::every].contiguous()
+    cfg_ref = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    k_ref = torch.cat([p[0].float() for p in past])
+    idx_ref = qwm.qwm_top1_keys(cfg_ref, qs, k_ref)
+    del k_ref
+    out = {}
+    variants = (("qvg", qwm.config(H, C, group_size=G, psac_rank=0, candidates=1), False, False),
+                ("qsac", qwm.config(H, C, group_size=G, psac_rank=0, candidates=M), True, False),
+                ("qsac_psac", cfg_ref, True, True))
+    for name, cfg, use_w, use_U in variants:
+        if name == "qsac_psac":
+            cache = hist
+        else:
+            cache = qwm.Cache(cfg, N, wl.past_chunks, device=dev)
+            for kd, vd, kc, vc, w, U in past:
+                qwm.qwm_quantize_append(cfg, cache, kd, vd, kc, vc, w=w if use_w else None, U=U if use_U else None)
+        k_hat = torch.cat([qwm.qwm_dequant_chunk(cfg, cache, i)[0] for i in range(cache.num_chunks)])
+        idx = qwm.qwm_top1_keys(cfg, qs, k_hat)
+        out[name] = round(float((idx != idx_ref).float().mean().item()), 4)
+        if cache.status():
+            raise RuntimeError(f"device status after the {name} cache")
+        del k_hat
+    out["queries"] = f"{qs.shape[0]} of {qd.shape[0]} (every {every}th) x {H} heads"
+    out["keys"] = int(sum(p[0].shape[0] for p in past))
+    out["reference"] = "bf16 keys, fp32 channel-order logits"
+    return out
 
 
 def fit_timing(qwm, cfg, kd, vd, ws, dev, iters, stream):

@@ -243,6 +243,28 @@ QWM_API qwm_status qwm_query_basis(const qwm_config* cfg, const void* stats, flo
  * word (*status) and read the Query count (*count, may be NULL). */
 QWM_API qwm_status qwm_query_stats_read(void* stats, int32_t* status, int64_t* count, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Token-selection shift measurement (Sec. 5, table "top1_shift": the share of
+ * queries whose highest-logit key changes when the cached Keys are quantized).
+ * --------------------------------------------------------------------------- */
+
+/* Reconstruction of cached chunk i (0 = oldest held; N = its token count from
+ * qwm_cache_chunk_info), the values attention rebuilds (App. D.1 on-demand
+ * reconstruction, Sec. 2 Eq. 3 and Sec. 4.2 Eq. 17):
+ * k_hat_c = mu_id,c + s_g (q_c - z_g) + sum_j t_j sigma U_r[c][j] for Keys (the PSAC
+ * term only when the chunk was stored with one), v_hat without it, in fp32
+ * (s (q - z) and t sigma exact, one fused multiply-add per PSAC term).
+ * k_out, v_out: fp32 [N][H][d], 16-byte aligned; either may be NULL. */
+QWM_API qwm_status qwm_dequant_chunk(const qwm_config* cfg, const qwm_cache* cache, int32_t i, float* k_out,
+                                     float* v_out, void* stream);
+
+/* Top-1 key of every query and head: idx[h][n] = argmax_j q[n,h] . keys[j,h],
+ * each logit the fp32 sum over channels in order with one fused multiply-add
+ * per term, ties to the lower key index.  q: bf16 [Nq][H][d]; keys: fp32
+ * [Nk][H][d] (16-byte aligned); idx: int32 [H][Nq].  Nq, Nk >= 1. */
+QWM_API qwm_status qwm_top1_keys(const qwm_config* cfg, const void* q, int64_t Nq, const float* keys, int64_t Nk,
+                                 int32_t* idx, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -11,9 +11,10 @@ Functions carry the C names:
   qwm_cache_bytes, qwm_fit_workspace_bytes, qwm_fit_centroids,
   qwm_fit_centroids_noalloc, qwm_quantize_append, qwm_attend,
 ``Cache`` wraps qwm_cache_init / qwm_cache_free / qwm_cache_status /
-qwm_cache_layout / qwm_cache_chunk_info, and ``QueryStats`` wraps a Query
+qwm_cache_layout / qwm_cache_chunk_info, ``QueryStats`` wraps a Query
 statistics buffer (qwm_query_stats_bytes / _reset / _update / _read and
-qwm_query_basis).
+qwm_query_basis), and qwm_dequant_chunk / qwm_top1_keys serve the
+token-selection shift measurement.
 """
 from __future__ import annotations
 
@@ -113,6 +114,10 @@ def lib():
             L.qwm_query_basis.restype = ct.c_int
             L.qwm_query_stats_read.argtypes = [_P, ct.POINTER(ct.c_int32), ct.POINTER(ct.c_int64), _P]
             L.qwm_query_stats_read.restype = ct.c_int
+            L.qwm_dequant_chunk.argtypes = [_CFG, _P, ct.c_int32, _P, _P, _P]
+            L.qwm_dequant_chunk.restype = ct.c_int
+            L.qwm_top1_keys.argtypes = [_CFG, _P, ct.c_int64, _P, ct.c_int64, _P, _P]
+            L.qwm_top1_keys.restype = ct.c_int
             _lib = L
     return _lib
 
@@ -372,3 +377,29 @@ class QueryStats:
     def sweeps(self) -> int:
         """Jacobi sweeps of the last basis computation (maximum over heads)."""
         return int(self.buffer[16:20].view(torch.int32).item())
+
+
+# ------------------------------------------------------------------ token-selection shift
+def qwm_dequant_chunk(cfg: QwmConfig, cache: Cache, i: int, keys=True, values=False):
+    """fp32 reconstruction of cached chunk i: (k_hat, v_hat), each [N][H][d] or None."""
+    _, N = cache.chunk_info(i)
+    H, d = cfg.num_heads, cfg.head_dim
+    dev = cache.buffer.device
+    k = torch.empty(N, H, d, dtype=torch.float32, device=dev) if keys else None
+    v = torch.empty(N, H, d, dtype=torch.float32, device=dev) if values else None
+    _check("qwm_dequant_chunk", lib().qwm_dequant_chunk(ct.byref(cfg), cache.handle, i, _ptr(k), _ptr(v),
+                                                        _stream()))
+    return k, v
+
+
+def qwm_top1_keys(cfg: QwmConfig, q, keys, idx=None):
+    """Index of the highest-logit key for every query and head, int32 [H][Nq]."""
+    Nq, Nk = q.shape[0], keys.shape[0]
+    H, d = cfg.num_heads, cfg.head_dim
+    _bf16(q, (Nq, H, d), "q")
+    if not (keys.is_cuda and keys.dtype == torch.float32 and keys.is_contiguous() and tuple(keys.shape) == (Nk, H, d)):
+        raise ValueError("keys must be a contiguous fp32 CUDA tensor [Nk][H][d]")
+    if idx is None:
+        idx = torch.empty(H, Nq, dtype=torch.int32, device=q.device)
+    _check("qwm_top1_keys", lib().qwm_top1_keys(ct.byref(cfg), _ptr(q), Nq, _ptr(keys), Nk, _ptr(idx), _stream()))
+    return idx

@@ -152,6 +152,28 @@ qwm_status qwm_cache_chunk_info(const qwm_cache* c, int32_t i, int32_t* slot, in
   return QWM_OK;
 }
 
+qwm_status qwm_dequant_chunk(const qwm_config* cfg, const qwm_cache* c, int32_t i, float* k_out, float* v_out,
+                             void* stream) {
+  if (!cfg || !c) return QWM_ERR_INVALID_ARG;
+  if (!supported(cfg)) return QWM_ERR_UNSUPPORTED;
+  if (!same_shape(cfg, &c->cfg)) return QWM_ERR_INVALID_ARG;
+  if ((k_out && !aligned16(k_out)) || (v_out && !aligned16(v_out))) return QWM_ERR_INVALID_ARG;
+  int32_t slot = 0;
+  int64_t tokens = 0;
+  const qwm_status st = qwm_cache_chunk_info(c, i, &slot, &tokens);
+  if (st != QWM_OK) return st;
+  if (!k_out && !v_out) return QWM_OK;
+  qwm::DequantArgs a{};
+  a.L = c->L;
+  a.base = c->base;
+  a.slot = slot;
+  a.N = tokens;
+  a.psac = c->psac[slot];
+  a.k_out = k_out;
+  a.v_out = v_out;
+  return qwm::launch_dequant(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
+}
+
 qwm_status qwm_cache_layout(const qwm_cache* c, qwm_layout* o) {
   if (!c || !o) return QWM_ERR_INVALID_ARG;
   const Layout& L = c->L;

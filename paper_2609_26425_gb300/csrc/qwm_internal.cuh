@@ -144,6 +144,17 @@ struct FitArgs {
   uint8_t* asg;                // [H][N] assignment
   int32_t* list;               // [H][N] member token indices grouped by cluster
 };
+struct DequantArgs {
+  Layout L;
+  const uint8_t* base;         // cache buffer
+  int slot;
+  int64_t N;                   // tokens in the chunk
+  int psac;                    // chunk stored with a PSAC correction
+  float* k_out;                // [N][H][d] fp32 or null
+  float* v_out;
+};
+cudaError_t launch_dequant(const DequantArgs& a, cudaStream_t s);
+
 // Byte size of the k-means workspace for H heads of N tokens and C centroids
 // (head_dim 128), and the carving of a workspace into FitArgs.
 size_t fit_workspace_bytes(int H, int d, int C, int64_t N);
