@@ -476,22 +476,39 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
     const int U = a.emax[h] - 134 - a.room;
     int64_t k0 = 0, k1 = 0, k2 = 0, k3 = 0;
     bool grid_ok = true;
-    // a member value in units of 2^U: (128 + f) << (e - 134 - U), below
-    // 2^(8 + room); zero stays zero; a value off the grid clears grid_ok
-    auto fix = [&](uint32_t b16) -> int64_t {
-      const uint32_t e = (b16 >> 7) & 0xFFu, f = b16 & 0x7Fu;
-      if (e == 0u) {
-        grid_ok = grid_ok && f == 0u;
-        return 0;
-      }
-      const int sh = (int)e - 134 - U;
-      grid_ok = grid_ok && sh >= 0 && e != 255u;
-      const int64_t v = (int64_t)(128u + f) << (sh & 63);
-      return (b16 & 0x8000u) ? -v : v;
+    // A member value in units of 2^U, y = (128 + f) 2^(e - 134 - U) < 2^48 (room <= 40),
+    // has 8 significant bits: the bf16 bits widened to fp32 with -U added to the
+    // exponent field.  Two additions of 3 2^54 and 3 2^38 split it exactly into
+    // fp32 limbs that are multiples of 2^32 and 2^16 and a remainder below
+    // 2^15; 32 such limbs add exactly in fp32 (below 2^21 units each), and every
+    // 32 members the three limb sums go to int64.  Zero stays zero; a value off
+    // the grid (tiny, subnormal, inf, NaN) clears grid_ok.
+    const uint32_t eadd = (uint32_t)(-U) << 23;
+    const int emin = U + 134;
+    const float C32 = 5.4043195528445952e16f;   // 3 * 2^54
+    const float C16 = 8.24633720832e11f;        // 3 * 2^38
+    float l2[4], l1[4], l0[4];
+    auto limb = [&](uint32_t b16, int ch) {
+      const uint32_t e = (b16 >> 7) & 0xFFu;
+      const bool zero = (b16 & 0x7FFFu) == 0u;
+      grid_ok = grid_ok && (zero || ((int)e >= emin && e != 255u));
+      const float y = zero ? 0.0f : __uint_as_float((b16 << 16) + eadd);
+      const float hi = __fsub_rn(__fadd_rn(y, C32), C32);
+      const float r1 = __fsub_rn(y, hi);
+      const float mid = __fsub_rn(__fadd_rn(r1, C16), C16);
+      l2[ch] = __fadd_rn(l2[ch], hi);
+      l1[ch] = __fadd_rn(l1[ch], mid);
+      l0[ch] = __fadd_rn(l0[ch], __fsub_rn(r1, mid));
+    };
+    auto flush = [&](int64_t& k, int ch) {
+      k += ((int64_t)__float2int_rn(l2[ch] * 2.3283064365386963e-10f) << 32) +
+           ((int64_t)__float2int_rn(l1[ch] * 1.52587890625e-05f) << 16) + (int64_t)__float2int_rn(l0[ch]);
     };
     for (int i0 = 0; i0 < cnt; i0 += 32) {
       const int nb = min(32, cnt - i0);
       const int my = lane < nb ? lst[i0 + lane] : -1;  // 32 member indices in one read
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) l2[ch] = l1[ch] = l0[ch] = 0.0f;
       for (int kb = 0; kb < nb; kb += 8) {
         uint2 xv[8];
 #pragma unroll
@@ -503,12 +520,16 @@ __global__ void __launch_bounds__(512) fit_means(const FitArgs a) {
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-          k0 += fix(xv[k].x & 0xFFFFu);
-          k1 += fix(xv[k].x >> 16);
-          k2 += fix(xv[k].y & 0xFFFFu);
-          k3 += fix(xv[k].y >> 16);
+          limb(xv[k].x & 0xFFFFu, 0);
+          limb(xv[k].x >> 16, 1);
+          limb(xv[k].y & 0xFFFFu, 2);
+          limb(xv[k].y >> 16, 3);
         }
       }
+      flush(k0, 0);
+      flush(k1, 1);
+      flush(k2, 2);
+      flush(k3, 3);
     }
     const double dc = (double)cnt;
     bool ok = __all_sync(0xFFFFFFFFu, grid_ok);
@@ -590,10 +611,11 @@ void fit_carve(FitArgs& a, uint8_t* ws) {
   a.nrm = reinterpret_cast<float*>(take((int64_t)a.H * a.Npad * 4));
   a.nmax = reinterpret_cast<uint32_t*>(take((int64_t)a.H * 4));
   a.emax = reinterpret_cast<int32_t*>(take((int64_t)a.H * 4));
-  // member sums of at most N values below 2^(8 + room) each stay below 2^61
+  // member sums of at most N values below 2^(8 + room) each stay below 2^61, and
+  // each value below 2^48 units
   int lg = 0;
   while (((int64_t)1 << lg) < a.N + 1) ++lg;
-  a.room = 53 - lg;
+  a.room = 53 - lg < 40 ? 53 - lg : 40;  // values below 2^48 units: three fp32 limbs (fit_means)
   a.counts = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.offs = reinterpret_cast<int32_t*>(take((int64_t)a.H * a.C * 4));
   a.asg = take((int64_t)a.H * a.N);
