@@ -77,3 +77,30 @@ def test_unsupported_shapes_size_to_zero(qlib):
     # centroids H*C*d*4, operand images H*P*512 (P = C rounded to 16), assignment and lists H*N*5
     assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 10) >= 4 * 64 * 128 * 4 + 4 * 64 * 512 + 4 * 10 * 5
     assert qlib.qwm_fit_workspace_bytes(qlib.config(4, 64), 20000) >= 4 * 64 * 128 * 4 + 4 * 64 * 512 + 4 * 20000 * 5
+
+
+def test_query_statistics_and_measurement_host_errors(qlib):
+    """Argument errors of the Query-statistics and measurement entry points come
+    back before anything touches a device (these calls never reach CUDA)."""
+    L = qlib.lib()
+    cfg = qlib.config(4, 64, psac_rank=16)
+    bad = qlib.config(4, 64, psac_rank=12)
+    fake = ct.c_void_p(1 << 20)            # 256-byte aligned, never dereferenced
+    unaligned = ct.c_void_p((1 << 20) + 8)
+    assert L.qwm_query_stats_bytes(ct.byref(cfg)) == 256 + 4 * 128 * 128 * 4
+    assert L.qwm_query_stats_bytes(ct.byref(bad)) == 0
+    assert L.qwm_query_stats_update(ct.byref(bad), fake, fake, 10, None) == 2
+    assert L.qwm_query_stats_update(ct.byref(cfg), None, fake, 10, None) == 1
+    assert L.qwm_query_stats_update(ct.byref(cfg), unaligned, fake, 10, None) == 1
+    assert L.qwm_query_stats_update(ct.byref(cfg), fake, fake, -1, None) == 1
+    assert L.qwm_query_stats_update(ct.byref(cfg), fake, None, 0, None) == 0     # N = 0: nothing to do
+    assert L.qwm_query_stats_update(ct.byref(cfg), fake, None, 5, None) == 1
+    assert L.qwm_query_basis(ct.byref(cfg), fake, None, None, None, None) == 0   # nothing requested
+    assert L.qwm_query_basis(ct.byref(bad), fake, None, None, None, None) == 2
+    assert L.qwm_query_basis(ct.byref(cfg), fake, ct.c_void_p((1 << 20) + 2), None, None, None) == 1
+    assert L.qwm_query_stats_read(None, None, None, None) == 1
+    assert L.qwm_top1_keys(ct.byref(cfg), fake, 0, fake, 10, fake, None) == 1
+    assert L.qwm_top1_keys(ct.byref(cfg), fake, 10, fake, 0, fake, None) == 1
+    assert L.qwm_top1_keys(ct.byref(bad), fake, 10, fake, 10, fake, None) == 2
+    assert L.qwm_top1_keys(ct.byref(cfg), fake, 10, ct.c_void_p((1 << 20) + 4), 10, fake, None) == 1
+    assert L.qwm_dequant_chunk(ct.byref(cfg), None, 0, fake, None, None) == 1
