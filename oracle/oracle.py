@@ -66,9 +66,9 @@ def _declare(L):
                                        _p, _p, _p, _p, ct.c_int]
     L.oracle_fit_centroids.restype = ct.c_int
     L.oracle_quantize.argtypes = ([ct.c_int] * 7 + [_p, ct.c_int64, _p, _p, _p, _p]
-                                  + [_p] * 7 + [_p] * 7 + [ct.c_int])
+                                  + [_p] * 7 + [_p] * 7 + [ct.c_int] + [ct.c_int, _p, _p])
     L.oracle_quantize.restype = ct.c_int
-    L.oracle_dequant.argtypes = [ct.c_int] * 5 + [ct.c_int64] + [_p] * 9
+    L.oracle_dequant.argtypes = [ct.c_int] * 5 + [ct.c_int64] + [_p] * 11
     L.oracle_dequant.restype = ct.c_int
     L.oracle_attend.argtypes = [ct.c_int, ct.c_int, ct.c_int64, ct.c_int64, _p, _p, _p,
                                 ct.c_double, _p, ct.c_int64, _p, _p, ct.c_int]
@@ -136,13 +136,18 @@ def fit_centroids(x_bits, C: int, iters: int, nthreads: int = 0):
 
 # ---------------------------------------------------------------- append
 def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
-             w=None, U_bits=None, force_ids=None, keep_scores: bool = False, nthreads: int = 0):
+             w=None, U_bits=None, force_ids=None, keep_scores: bool = False, nthreads: int = 0,
+             two_level_scales: bool = False):
     """QSAC + INT2 + PSAC for one chunk (see oracle_quantize).
 
     x_bits uint16 [N][H][d]; cent_bits uint16 [H][C][d]; w float32 [H][d] or
     None; U_bits uint16 [H][d][r] or None.  Returns a dict of token-major
     arrays: ids, codes, scales, zeros, coef, sigma, kept, khat0, cand,
     m_topm, m_sel, m_psac and, with keep_scores, dq [N][H][C] and S [N][H][M'].
+    two_level_scales: the App. D.1 storage of group scales (uint8 codes with
+    one binary16 secondary scale per token-head, see two_level_scales in the
+    C source); adds scode [N][H][d/G] and s2 [N][H] (binary16 bits), and the
+    binary16 scales are left zero.
     """
     x = _c(x_bits, np.uint16)
     cent = _c(cent_bits, np.uint16)
@@ -170,6 +175,8 @@ def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
         "m_psac": np.ones((N, H), np.float32),
         "dq": np.zeros((N, H, C), np.float32) if keep_scores else None,
         "S": np.zeros((N, H, Mc), np.float32) if keep_scores else None,
+        "scode": np.zeros((N, H, ng), np.uint8) if two_level_scales else None,
+        "s2": np.zeros((N, H), np.uint16) if two_level_scales else None,
     }
     if N == 0:
         return o
@@ -177,7 +184,8 @@ def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
         H, d, C, G, r, M, int(bool(is_key)), _ptr(x), N, _ptr(cent), _ptr(wv), _ptr(Uv), _ptr(fid),
         _ptr(o["ids"]), _ptr(o["codes"]), _ptr(o["scales"]), _ptr(o["zeros"]), _ptr(o["coef"]),
         _ptr(o["sigma"]), _ptr(o["kept"]), _ptr(o["khat0"]), _ptr(o["cand"]), _ptr(o["m_topm"]),
-        _ptr(o["m_sel"]), _ptr(o["m_psac"]), _ptr(o["dq"]), _ptr(o["S"]), nthreads)
+        _ptr(o["m_sel"]), _ptr(o["m_psac"]), _ptr(o["dq"]), _ptr(o["S"]), nthreads,
+        1 if two_level_scales else 0, _ptr(o["scode"]), _ptr(o["s2"]))
     if rc:
         raise ValueError(f"oracle_quantize: invalid arguments (rc={rc})")
     return o
@@ -197,7 +205,8 @@ def dequant(q, cent_bits, *, G: int, r: int, U_bits=None):
     rc = lib().oracle_dequant(H, d, C, G, r if use_psac else 0, N, _ptr(cent), _ptr(ids),
                               _ptr(_c(q["codes"], np.uint8)), _ptr(_c(q["scales"], np.uint16)),
                               _ptr(_c(q["zeros"], np.uint8)), _ptr(coef), _ptr(sig), _ptr(Uv),
-                              _ptr(out))
+                              _ptr(out), _ptr(None if q.get("scode") is None else _c(q["scode"], np.uint8)),
+                              _ptr(None if q.get("s2") is None else _c(q["s2"], np.uint16)))
     if rc:
         raise ValueError(f"oracle_dequant: invalid arguments (rc={rc})")
     return out
@@ -283,3 +292,17 @@ def top1(q_bits, k):
 def top1_shift(idx_ref, idx):
     """Share of (query, head) pairs whose top-1 key differs from the reference's."""
     return float(np.mean(np.asarray(idx_ref) != np.asarray(idx)))
+
+
+# ---------------------------------------------------------------- storage accounting
+def psac_layout_bytes(kept, r: int, N: int | None = None):
+    """Bytes of one chunk-head's PSAC coefficients in the two layouts App. D.1
+    chooses between (reading: dense = every row's r INT8 codes and binary16
+    scale; sparse = the kept rows only, each with a uint16 token index, plus a
+    4-byte row count).  kept: bool/uint8 [N].  Returns (dense, sparse, chosen)."""
+    kept = np.asarray(kept).astype(bool)
+    n = kept.size if N is None else N
+    K = int(kept.sum())
+    dense = n * (r + 2)
+    sparse = K * (r + 2 + 2) + 4
+    return dense, sparse, min(dense, sparse)

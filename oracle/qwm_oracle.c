@@ -239,16 +239,32 @@ static float rel_gap(float a, float b) {
  * x * (1/s); rounding is half to even; an all-zero range gives s = 0, z = 0,
  * codes 0.
  */
-static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uint8_t* q_out) {
+/* The zero-inclusive range of a group over 3 (the scale before storage). */
+static float group_s32(const float* xg, int G) {
   float lo = 0.0f, hi = 0.0f;
   for (int c = 0; c < G; ++c) {
     if (xg[c] < lo) lo = xg[c];
     if (xg[c] > hi) hi = xg[c];
   }
-  float s32 = (hi - lo) / 3.0f;
+  return (hi - lo) / 3.0f;
+}
+
+/* Codes and zero-point of one group for a given stored scale s (>= the
+ * group's (hi - lo) / 3, so the three steps still span the range). */
+static void int2_group_with(const float* xg, int G, float s, int* z_out, uint8_t* q_out);
+
+static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uint8_t* q_out) {
+  float s32 = group_s32(xg, G);
   uint16_t sb = oracle_f32_to_f16_ru(s32);
   float s = oracle_f16_to_f32(sb);
   *s_bits = sb;
+  int2_group_with(xg, G, s, z_out, q_out);
+}
+
+static void int2_group_with(const float* xg, int G, float s, int* z_out, uint8_t* q_out) {
+  float lo = 0.0f;
+  for (int c = 0; c < G; ++c)
+    if (xg[c] < lo) lo = xg[c];
   if (s == 0.0f) {
     *z_out = 0;
     for (int c = 0; c < G; ++c) q_out[c] = 0;
@@ -265,6 +281,43 @@ static void int2_group(const float* xg, int G, uint16_t* s_bits, int* z_out, uin
     if (q < 0) q = 0;
     if (q > 3) q = 3;
     q_out[c] = (uint8_t)q;
+  }
+}
+
+/*
+ * Two-level group scales (App. D.1: "group scales use INT8 codes with a
+ * shared FP16 secondary scale").  Readings: the secondary scale is shared by
+ * the d/G groups of one token-head; s2 = binary16 round-up of
+ * max_g s32_g / 255 with s32_g = (hi_g - lo_g) / 3 (reading 2's range); each
+ * group's code is the smallest integer c in [0, 255] with c * s2 >= s32_g (an
+ * unsigned byte: scales are never negative); the stored scale c * s2 (exact
+ * in fp32) then quantizes the group, so the step still covers the range.
+ */
+static void two_level_scales(const float* res, int d, int G, uint8_t* code, uint16_t* s2_bits, float* s_eff) {
+  const int ng = d / G;
+  float mx = 0.0f;
+  float s32[64];
+  for (int g = 0; g < ng; ++g) {
+    s32[g] = group_s32(res + g * G, G);
+    if (s32[g] > mx) mx = s32[g];
+  }
+  uint16_t sb = oracle_f32_to_f16_ru(mx / 255.0f);
+  float s2 = oracle_f16_to_f32(sb);
+  if (mx > 0.0f && 255.0f * s2 < mx) {   /* mx / 255 rounded down in fp32: one binary16 step up */
+    sb = (uint16_t)(sb + 1);
+    s2 = oracle_f16_to_f32(sb);
+  }
+  *s2_bits = sb;
+  for (int g = 0; g < ng; ++g) {
+    int c = 0;
+    if (s2 > 0.0f) {
+      c = (int)ceilf(s32[g] / s2);
+      if (c > 0 && (float)(c - 1) * s2 >= s32[g]) c -= 1;   /* smallest covering code */
+      if ((float)c * s2 < s32[g]) c += 1;
+      if (c > 255) c = 255;
+    }
+    code[g] = (uint8_t)c;
+    s_eff[g] = (float)c * s2;
   }
 }
 
@@ -322,10 +375,12 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
                     uint8_t* ids, uint8_t* codes, uint16_t* scales, uint8_t* zeros,
                     int8_t* coef, uint16_t* sigma, uint8_t* kept,
                     float* khat0, int32_t* cand, float* m_topm, float* m_sel, float* m_psac,
-                    float* dq_out, float* s_out, int nthreads) {
+                    float* dq_out, float* s_out, int nthreads,
+                    int scale_mode, uint8_t* scode, uint16_t* s2) {
   if (H <= 0 || d <= 0 || d > 256 || C <= 0 || C > 256 || G <= 0 || d % G || d % 16 || r < 0 || M <= 0 || N < 0)
     return ORC_EINVAL;
   if (!x || !cent || !ids || !codes || !scales || !zeros) return ORC_EINVAL;
+  if (scale_mode != 0 && (scale_mode != 1 || !scode || !s2 || d / G > 64)) return ORC_EINVAL;
   const int ng = d / G;
   const int zb = (2 * ng + 7) / 8;
   const int Mc = M < C ? M : C;
@@ -442,13 +497,22 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
     uint8_t qv[256];
     for (int c = 0; c < d; ++c) res[c] = k[c] - oracle_bf16_to_f32(mu[c]);
     float* k0 = E; /* reuse: holds k0 first, then E */
+    float s_eff[64];
+    if (scale_mode == 1)
+      two_level_scales(res, d, G, scode + ((size_t)i * H + h) * ng, s2 + (size_t)i * H + h, s_eff);
     for (int g = 0; g < ng; ++g) {
-      uint16_t sb;
+      uint16_t sb = 0;
       int z;
-      int2_group(res + g * G, G, &sb, &z, qv);
+      float s;
+      if (scale_mode == 1) {
+        s = s_eff[g];
+        int2_group_with(res + g * G, G, s, &z, qv);
+      } else {
+        int2_group(res + g * G, G, &sb, &z, qv);
+        s = oracle_f16_to_f32(sb);
+      }
       sc[g] = sb;
       zz[g / 4] |= (uint8_t)(z << (2 * (g % 4)));
-      float s = oracle_f16_to_f32(sb);
       for (int c = g * G; c < (g + 1) * G; ++c) {
         int q = qv[c - g * G];
         int bit = code_bit(c);
@@ -542,7 +606,7 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
 int oracle_dequant(int H, int d, int C, int G, int r, int64_t N, const uint16_t* cent,
                    const uint8_t* ids, const uint8_t* codes, const uint16_t* scales,
                    const uint8_t* zeros, const int8_t* coef, const uint16_t* sigma,
-                   const uint16_t* U, double* out) {
+                   const uint16_t* U, double* out, const uint8_t* scode, const uint16_t* s2) {
   if (H <= 0 || d <= 0 || C <= 0 || G <= 0 || d % G || N < 0 || !out) return ORC_EINVAL;
   const int ng = d / G;
   const int zb = (2 * ng + 7) / 8;
@@ -558,7 +622,8 @@ int oracle_dequant(int H, int d, int C, int G, int r, int64_t N, const uint16_t*
         int bit = code_bit(c);
         int q = (codes[th * (d / 4) + bit / 8] >> (bit % 8)) & 3;
         int z = (zeros[th * zb + g / 4] >> (2 * (g % 4))) & 3;
-        double s = (double)oracle_f16_to_f32(scales[th * ng + g]);
+        double s = scode ? (double)scode[th * ng + g] * (double)oracle_f16_to_f32(s2[th])
+                         : (double)oracle_f16_to_f32(scales[th * ng + g]);
         double v = (double)oracle_bf16_to_f32(mu[c]) + s * (double)(q - z);
         if (psac) {
           double sg = (double)oracle_f16_to_f32(sigma[th]);

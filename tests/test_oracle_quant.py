@@ -10,6 +10,7 @@ import os
 
 import numpy as np
 import pytest
+import torch
 from scipy.spatial.distance import cdist
 
 from paper_2609_26425_gb300 import synth
@@ -338,3 +339,68 @@ def test_psac_keep_rule_and_projection(orc):
     a = np.abs(c).max(-1) / 127
     sg = f16(o["sigma"])
     assert np.all(sg[kept] >= a[kept] * (1 - 1e-5))
+
+
+
+# ------------------------------------------------------------------ two-level group scales (App. D.1)
+def _one_token_chunk(groups):
+    """A single token of one head whose residual (centroid 0) has the given
+    32-channel groups; values are exact in bf16."""
+    k = np.concatenate([np.asarray(g, np.float32) for g in groups])[None, None, :]
+    kb = synth.bits(torch.from_numpy(k).to(torch.bfloat16))
+    cent = np.zeros((1, 1, 128), np.uint16)
+    return kb, cent
+
+
+def test_two_level_scales_hand_fixture(orc):
+    """Group ranges 3, 6, 1.5 and 0 give s32 = 1, 2, 0.5, 0; the secondary
+    scale is the binary16 round-up of 2/255 = 0.00784313...: 2^-7 + 5 * 2^-17
+    = 0.00785064697265625 (the binary16 step above 2^-7 is 2^-17); the codes
+    are ceil(s32 / s2) = 128, 255, 64, 0 (hand computed: 127.38, 254.76,
+    63.69)."""
+    g0 = np.tile([-1.5, 1.5], 16)
+    g1 = np.tile([0.0, 6.0], 16)
+    g2 = np.tile([-0.75, 0.75], 16)
+    g3 = np.zeros(32)
+    kb, cent = _one_token_chunk([g0, g1, g2, g3])
+    o = orc.quantize(kb, cent, G=32, r=0, M=1, is_key=True, two_level_scales=True)
+    s2 = float(orc.f16_to_f32(o["s2"])[0, 0])
+    assert s2 == 2.0 ** -7 + 5 * 2.0 ** -17
+    assert o["scode"][0, 0].tolist() == [128, 255, 64, 0]
+    assert np.all(o["scales"] == 0)
+
+
+def test_two_level_scales_cover_minimal_and_round_trip(orc):
+    """On random Keys: every code is the smallest with code * s2 >= the
+    group's (hi - lo) / 3, and the reconstruction keeps the INT2 bound
+    |x - x_hat| <= s / 2 with the stored scale s = code * s2."""
+    H, N, C, G = 2, 200, 16, 32
+    kb = synth.bits(synth.gaussian_bf16(41, N, H, 128, scale=2.0))
+    cent = synth.bits(synth.gaussian_bf16(42, H, C, 128))
+    o = orc.quantize(kb, cent, G=G, r=0, M=2, is_key=True, two_level_scales=True)
+    x = orc.bf16_to_f32(kb).astype(np.float64)
+    mu = orc.bf16_to_f32(cent).astype(np.float64)
+    s2 = orc.f16_to_f32(o["s2"]).astype(np.float64)
+    khat = orc.dequant(o, cent, G=G, r=0)
+    for i in range(N):
+        for h in range(H):
+            res = x[i, h] - mu[h, o["ids"][i, h]]
+            for g in range(128 // G):
+                rg = res[g * G:(g + 1) * G]
+                s32 = np.float32((np.float32(max(rg.max(), 0.0)) - np.float32(min(rg.min(), 0.0))) / np.float32(3.0))
+                c = int(o["scode"][i, h, g])
+                assert c * s2[i, h] >= s32 and (c == 0 or (c - 1) * s2[i, h] < s32)
+                step = c * s2[i, h]
+                assert np.all(np.abs(khat[i, h, g * G:(g + 1) * G] - x[i, h, g * G:(g + 1) * G]) <= step / 2 + 1e-12)
+
+
+def test_two_level_scales_zero_token_and_psac_layout(orc):
+    kb, cent = _one_token_chunk([np.zeros(32)] * 4)
+    o = orc.quantize(kb, cent, G=32, r=0, M=1, is_key=True, two_level_scales=True)
+    assert o["s2"][0, 0] == 0 and np.all(o["scode"] == 0) and np.all(o["codes"] == 0)
+    # App. D.1 layout choice, reading: dense N (r + 2) bytes, sparse K (r + 4) + 4
+    kept = np.zeros(100, bool)
+    kept[:10] = True
+    assert orc.psac_layout_bytes(kept, 8) == (1000, 124, 124)
+    kept[:] = True
+    assert orc.psac_layout_bytes(kept, 8) == (1000, 1204, 1000)
