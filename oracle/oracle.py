@@ -66,7 +66,7 @@ def _declare(L):
                                        _p, _p, _p, _p, ct.c_int]
     L.oracle_fit_centroids.restype = ct.c_int
     L.oracle_quantize.argtypes = ([ct.c_int] * 7 + [_p, ct.c_int64, _p, _p, _p, _p]
-                                  + [_p] * 7 + [_p] * 7 + [ct.c_int] + [ct.c_int, _p, _p])
+                                  + [_p] * 7 + [_p] * 7 + [ct.c_int] + [ct.c_int, _p, _p, _p])
     L.oracle_quantize.restype = ct.c_int
     L.oracle_dequant.argtypes = [ct.c_int] * 5 + [ct.c_int64] + [_p] * 11
     L.oracle_dequant.restype = ct.c_int
@@ -137,7 +137,7 @@ def fit_centroids(x_bits, C: int, iters: int, nthreads: int = 0):
 # ---------------------------------------------------------------- append
 def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
              w=None, U_bits=None, force_ids=None, keep_scores: bool = False, nthreads: int = 0,
-             two_level_scales: bool = False):
+             two_level_scales: bool = False, M_full=None):
     """QSAC + INT2 + PSAC for one chunk (see oracle_quantize).
 
     x_bits uint16 [N][H][d]; cent_bits uint16 [H][C][d]; w float32 [H][d] or
@@ -148,6 +148,9 @@ def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
     one binary16 secondary scale per token-head, see two_level_scales in the
     C source); adds scode [N][H][d/G] and s2 [N][H] (binary16 bits), and the
     binary16 scales are left zero.
+    M_full: float32 [H][d][d] or None; for Keys, the top-M candidates come from
+    the full quadratic form (k - mu)^T M (k - mu) instead of Eq. 9 (the
+    ablation of App. C.4); the QSAC score and everything after still use w.
     """
     x = _c(x_bits, np.uint16)
     cent = _c(cent_bits, np.uint16)
@@ -185,7 +188,8 @@ def quantize(x_bits, cent_bits, *, G: int, r: int, M: int, is_key: bool,
         _ptr(o["ids"]), _ptr(o["codes"]), _ptr(o["scales"]), _ptr(o["zeros"]), _ptr(o["coef"]),
         _ptr(o["sigma"]), _ptr(o["kept"]), _ptr(o["khat0"]), _ptr(o["cand"]), _ptr(o["m_topm"]),
         _ptr(o["m_sel"]), _ptr(o["m_psac"]), _ptr(o["dq"]), _ptr(o["S"]), nthreads,
-        1 if two_level_scales else 0, _ptr(o["scode"]), _ptr(o["s2"]))
+        1 if two_level_scales else 0, _ptr(o["scode"]), _ptr(o["s2"]),
+        _ptr(None if M_full is None else _c(M_full, np.float32)))
     if rc:
         raise ValueError(f"oracle_quantize: invalid arguments (rc={rc})")
     return o

@@ -376,7 +376,7 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
                     int8_t* coef, uint16_t* sigma, uint8_t* kept,
                     float* khat0, int32_t* cand, float* m_topm, float* m_sel, float* m_psac,
                     float* dq_out, float* s_out, int nthreads,
-                    int scale_mode, uint8_t* scode, uint16_t* s2) {
+                    int scale_mode, uint8_t* scode, uint16_t* s2, const float* Mfull) {
   if (H <= 0 || d <= 0 || d > 256 || C <= 0 || C > 256 || G <= 0 || d % G || d % 16 || r < 0 || M <= 0 || N < 0)
     return ORC_EINVAL;
   if (!x || !cent || !ids || !codes || !scales || !zeros) return ORC_EINVAL;
@@ -413,14 +413,27 @@ int oracle_quantize(int H, int d, int C, int G, int r, int M, int is_key,
       if (m_topm) m_topm[(size_t)i * H + h] = 1.0f;
       if (m_sel) m_sel[(size_t)i * H + h] = 1.0f;
     } else {
-      /* 1. Query-aware distance (Eq. 9) */
+      /* 1. Query-aware distance (Eq. 9), or with Mfull the full quadratic
+       * form of the ablation in App. C.4: e = k - mu_j (each difference
+       * rounded), t = M e (t_c = sum_c' M_cc' e_c', one fma per term in c'
+       * order), d = sum_c e_c t_c (one fma per term in c order). */
       for (int j = 0; j < C; ++j) {
         const uint16_t* mu = mu_h + (size_t)j * d;
         float acc = 0.0f;
-        for (int c = 0; c < d; ++c) {
-          float t = k[c] - oracle_bf16_to_f32(mu[c]);
-          float t2 = t * t;
-          acc = fmaf(wv[c], t2, acc); /* one fused multiply-add per term */
+        if (Mfull && is_key) {
+          const float* Mh = Mfull + (size_t)h * d * d;
+          for (int c = 0; c < d; ++c) res[c] = k[c] - oracle_bf16_to_f32(mu[c]);
+          for (int c = 0; c < d; ++c) {
+            float tc = 0.0f;
+            for (int c2 = 0; c2 < d; ++c2) tc = fmaf(Mh[(size_t)c * d + c2], res[c2], tc);
+            acc = fmaf(res[c], tc, acc);
+          }
+        } else {
+          for (int c = 0; c < d; ++c) {
+            float t = k[c] - oracle_bf16_to_f32(mu[c]);
+            float t2 = t * t;
+            acc = fmaf(wv[c], t2, acc); /* one fused multiply-add per term */
+          }
         }
         dq[j] = acc;
         chosen[j] = 0;

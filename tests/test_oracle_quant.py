@@ -404,3 +404,37 @@ def test_two_level_scales_zero_token_and_psac_layout(orc):
     assert orc.psac_layout_bytes(kept, 8) == (1000, 124, 124)
     kept[:] = True
     assert orc.psac_layout_bytes(kept, 8) == (1000, 1204, 1000)
+
+
+
+# ------------------------------------------------------------------ full-matrix distance (App. C.4 ablation)
+def test_full_matrix_distance_reduces_to_diagonal_and_matches_fp64(orc):
+    """With M = diag(w) the full quadratic form is Eq. 9's diagonal distance:
+    same candidates and ids wherever the decision margins are clear.  With a
+    dense symmetric positive M, the candidates are the M smallest fp64 values
+    of (k - mu)^T M (k - mu) (brute force) wherever the margin is clear."""
+    H, N, C, G, Mc = 2, 60, 16, 32, 4
+    kb = synth.bits(synth.gaussian_bf16(51, N, H, 128))
+    cent = synth.bits(synth.gaussian_bf16(52, H, C, 128))
+    w = synth.random_weights(53, H, 128).numpy()
+    Md = np.stack([np.diag(w[h]) for h in range(H)]).astype(np.float32)
+    a = orc.quantize(kb, cent, G=G, r=0, M=Mc, is_key=True, w=w)
+    b = orc.quantize(kb, cent, G=G, r=0, M=Mc, is_key=True, w=w, M_full=Md)
+    clear = (a["m_topm"] > 1e-5) & (b["m_topm"] > 1e-5) & (a["m_sel"] > 1e-5)
+    assert clear.mean() > 0.9
+    assert np.array_equal(np.sort(a["cand"], -1)[clear], np.sort(b["cand"], -1)[clear])
+    assert np.array_equal(a["ids"][clear], b["ids"][clear])
+    rng = np.random.default_rng(54)
+    R = rng.standard_normal((H, 128, 128))
+    Mf = (np.einsum("hij,hkj->hik", R, R) / 128).astype(np.float32)
+    c = orc.quantize(kb, cent, G=G, r=0, M=Mc, is_key=True, w=w, M_full=Mf)
+    x = orc.bf16_to_f32(kb).astype(np.float64)
+    mu = orc.bf16_to_f32(cent).astype(np.float64)
+    for i in range(N):
+        for h in range(H):
+            e = x[i, h][None, :] - mu[h]
+            dfull = np.einsum("jc,cd,jd->j", e, Mf[h].astype(np.float64), e)
+            order = np.argsort(dfull, kind="stable")
+            gap = (dfull[order[Mc]] - dfull[order[Mc - 1]]) / abs(dfull[order[Mc]])
+            if gap > 1e-4:
+                assert set(c["cand"][i, h]) == set(order[:Mc])
