@@ -29,8 +29,8 @@
  *     word, read with qwm_cache_status.
  *   - Supported: head_dim 128; group_size 32 or 64; 1 <= num_centroids <= 256;
  *     psac_rank 0, 8, 16 or 32; num_candidates >= 1 (values above
- *     num_centroids mean "all centroids").  Anything else returns
- *     QWM_ERR_UNSUPPORTED.
+ *     num_centroids mean "all centroids"); scale_format 0 or 1.  Anything
+ *     else returns QWM_ERR_UNSUPPORTED.
  */
 #ifndef QWM_H
 #define QWM_H
@@ -59,6 +59,10 @@ typedef struct qwm_config {
   int32_t psac_rank;
   int32_t num_candidates;
   int32_t kmeans_iters;
+  /* Storage of the INT2 group scales: 0 = one binary16 per group; 1 = App. D.1's
+   * uint8 code per group with one binary16 secondary scale per token-head
+   * (the group's scale is code * secondary).  Zero-initialise the struct. */
+  int32_t scale_format;
 } qwm_config;
 
 typedef enum qwm_status {
@@ -82,7 +86,9 @@ typedef struct qwm_cache qwm_cache;
  * structure-of-arrays fields (offsets within the tile): codes [128][d/4] u8
  * (channel c in byte c/4, bits 2(c%4)), scales [128][d/G] binary16,
  * ids [128] u8, zero-points [128][zb] u8 (group g in byte g/4, bits 2(g%4)),
- * and for Keys PSAC codes [128][r] int8 and row scales [128] binary16. */
+ * and for Keys PSAC codes [128][r] int8 and row scales [128] binary16.  With
+ * scale_format 1 the scale field holds [128][d/G] u8 codes and a secondary
+ * scale field [128] binary16 follows it (k_s2, v_s2). */
 typedef struct qwm_layout {
   int64_t header_bytes;     /* device status word + reserved, before slot 0 */
   int64_t slot_meta_bytes;  /* per-slot reserved bytes before head 0 */
@@ -93,6 +99,8 @@ typedef struct qwm_layout {
   int64_t k_codes, k_scales, k_ids, k_zeros, k_coef, k_sigma, k_bytes; /* within a tile */
   int64_t v_codes, v_scales, v_ids, v_zeros, v_bytes; /* within a tile, from its start */
   int64_t zero_bytes;       /* zb: bytes of packed zero-points per token */
+  int64_t k_s2, v_s2;       /* scale_format 1: secondary scales [128] binary16 (k_scales, v_scales
+                               then hold [128][d/G] uint8 codes); 0 otherwise */
 } qwm_layout;
 
 /* Human-readable name of a status code (static string). */

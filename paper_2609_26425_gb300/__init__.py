@@ -43,16 +43,17 @@ class QwmError(RuntimeError):
 class QwmConfig(ct.Structure):
     _fields_ = [("num_heads", ct.c_int32), ("head_dim", ct.c_int32), ("num_centroids", ct.c_int32),
                 ("group_size", ct.c_int32), ("psac_rank", ct.c_int32), ("num_candidates", ct.c_int32),
-                ("kmeans_iters", ct.c_int32)]
+                ("kmeans_iters", ct.c_int32), ("scale_format", ct.c_int32)]
 
     def __repr__(self):
-        return ("QwmConfig(H=%d, d=%d, C=%d, G=%d, r=%d, M=%d, iters=%d)" %
+        return ("QwmConfig(H=%d, d=%d, C=%d, G=%d, r=%d, M=%d, iters=%d, scale_format=%d)" %
                 (self.num_heads, self.head_dim, self.num_centroids, self.group_size, self.psac_rank,
-                 self.num_candidates, self.kmeans_iters))
+                 self.num_candidates, self.kmeans_iters, self.scale_format))
 
 
-def config(heads, centroids, group_size=32, psac_rank=16, candidates=4, kmeans_iters=10, head_dim=128):
-    return QwmConfig(heads, head_dim, centroids, group_size, psac_rank, candidates, kmeans_iters)
+def config(heads, centroids, group_size=32, psac_rank=16, candidates=4, kmeans_iters=10, head_dim=128,
+           scale_format=0):
+    return QwmConfig(heads, head_dim, centroids, group_size, psac_rank, candidates, kmeans_iters, scale_format)
 
 
 class QwmLayout(ct.Structure):
@@ -61,7 +62,7 @@ class QwmLayout(ct.Structure):
         "ktab_offset", "vtab_offset", "ut_offset", "tiles_offset",
         "tile_tokens", "tiles_per_chunk", "tile_bytes",
         "k_codes", "k_scales", "k_ids", "k_zeros", "k_coef", "k_sigma", "k_bytes",
-        "v_codes", "v_scales", "v_ids", "v_zeros", "v_bytes", "zero_bytes")]
+        "v_codes", "v_scales", "v_ids", "v_zeros", "v_bytes", "zero_bytes", "k_s2", "v_s2")]
 
 
 _lib = None
@@ -205,7 +206,9 @@ class Cache:
         arrays (layout only; no arithmetic): ids [N][H], codes [N][H][d/4],
         scales [N][H][d/G] (binary16 bits), zeros [N][H][zb], coef [N][H][r],
         sigma [N][H] (binary16 bits), k_tab / v_tab [H][C][d] (binary16 bits,
-        the tables as stored in the slot) and U [H][d][r] (bf16 bits)."""
+        the tables as stored in the slot) and U [H][d][r] (bf16 bits).  With
+        scale_format 1, scode [N][H][d/G] u8 and s2 [N][H] (binary16 bits)
+        replace scales (and v_scode, v_s2 for Values)."""
         slot, N = self.chunk_info(i)
         lay = self.layout()
         cfg = self.cfg
@@ -215,8 +218,10 @@ class Cache:
         raw = self.buffer[start:start + lay.slot_bytes].cpu().numpy()
         T = lay.tile_tokens
         ntile = (N + T - 1) // T
-        out = {k: [] for k in ("ids", "codes", "scales", "zeros", "coef", "sigma",
-                               "v_ids", "v_codes", "v_scales", "v_zeros")}
+        sf = cfg.scale_format
+        keys = ("ids", "codes", "zeros", "coef", "sigma", "v_ids", "v_codes", "v_zeros")
+        keys += ("scode", "s2", "v_scode", "v_s2") if sf else ("scales", "v_scales")
+        out = {k: [] for k in keys}
         k_tab = np.zeros((H, C, d), np.uint16)
         v_tab = np.zeros((H, C, d), np.uint16)
         U = np.zeros((H, d, r), np.uint16)
@@ -234,13 +239,19 @@ class Cache:
                 return np.ascontiguousarray(b).view(dtype)
 
             out["codes"].append(f(lay.k_codes, d // 4))
-            out["scales"].append(f(lay.k_scales, ng * 2, np.uint16))
+            if sf:
+                out["scode"].append(f(lay.k_scales, ng))
+                out["s2"].append(f(lay.k_s2, 2, np.uint16)[:, 0])
+                out["v_scode"].append(f(lay.v_scales, ng))
+                out["v_s2"].append(f(lay.v_s2, 2, np.uint16)[:, 0])
+            else:
+                out["scales"].append(f(lay.k_scales, ng * 2, np.uint16))
+                out["v_scales"].append(f(lay.v_scales, ng * 2, np.uint16))
             out["ids"].append(f(lay.k_ids, 1)[:, 0])
             out["zeros"].append(f(lay.k_zeros, zb))
             out["coef"].append(f(lay.k_coef, r, np.int8) if r else np.zeros((N, 0), np.int8))
             out["sigma"].append(f(lay.k_sigma, 2, np.uint16)[:, 0] if r else np.zeros(N, np.uint16))
             out["v_codes"].append(f(lay.v_codes, d // 4))
-            out["v_scales"].append(f(lay.v_scales, ng * 2, np.uint16))
             out["v_ids"].append(f(lay.v_ids, 1)[:, 0])
             out["v_zeros"].append(f(lay.v_zeros, zb))
         res = {k: np.stack(v, axis=1) for k, v in out.items()}

@@ -624,6 +624,8 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
     const __nv_bfloat16* mr = tab;
     float sc[4], inv[4], zf[4];
     __half sh[4];
+    uint32_t scode[4] = {0u, 0u, 0u, 0u};   // scale format 1: group codes and secondary scale
+    __half s2h = __ushort_as_half(0);
     uint32_t zbyte = 0;
     uint64_t cj[RP], vj[RP];
 #pragma unroll
@@ -792,14 +794,47 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
       id = bestj < C ? bestj : C - 1;
       mr = tab + (size_t)id * 128;
 
-      // ---- 3. INT2 parameters (Eq. 1-2): range of the residual with 0 included
+      // ---- 3. INT2 parameters (Eq. 1-2): range of the residual with 0 included;
+      // scale format 1 (App. D.1): s = code * s2 with s2 the binary16 round-up of
+      // max_g range_g / 3 / 255 and code the smallest byte covering range_g / 3
+      float s32g[4];
+      float smax = 0.0f;
+    #pragma unroll
+      for (int gi = 0; gi < 4; ++gi) {
+        s32g[gi] = 0.0f;
+        if (gi < ng) {
+          s32g[gi] = __fdiv_rn(__fsub_rn(fmaxf(0.0f, bmx[gi]), fminf(0.0f, bmn[gi])), 3.0f);
+          smax = fmaxf(smax, s32g[gi]);
+        }
+      }
+      float s2f = 0.0f;
+      if (L.sf) {
+        s2h = __float2half_ru(__fdiv_rn(smax, 255.0f));
+        s2f = __half2float(s2h);
+        if (smax > 0.0f && __fmul_rn(255.0f, s2f) < smax) {
+          s2h = __ushort_as_half((unsigned short)(__half_as_ushort(s2h) + 1));
+          s2f = __half2float(s2h);
+        }
+      }
     #pragma unroll
       for (int gi = 0; gi < 4; ++gi) {
         sc[gi] = 0.0f; inv[gi] = 0.0f; zf[gi] = 0.0f; sh[gi] = __ushort_as_half(0);
         if (gi < ng) {
-          const float lo = fminf(0.0f, bmn[gi]), hi = fmaxf(0.0f, bmx[gi]);
-          sh[gi] = __float2half_ru(__fdiv_rn(__fsub_rn(hi, lo), 3.0f));
-          sc[gi] = __half2float(sh[gi]);
+          const float lo = fminf(0.0f, bmn[gi]);
+          if (L.sf) {
+            int c = 0;
+            if (s2f > 0.0f) {
+              c = (int)ceilf(__fdiv_rn(s32g[gi], s2f));
+              if (c > 0 && __fmul_rn((float)(c - 1), s2f) >= s32g[gi]) c -= 1;
+              if (__fmul_rn((float)c, s2f) < s32g[gi]) c += 1;
+              c = c > 255 ? 255 : c;
+            }
+            scode[gi] = (uint32_t)c;
+            sc[gi] = __fmul_rn((float)c, s2f);
+          } else {
+            sh[gi] = __float2half_ru(s32g[gi]);
+            sc[gi] = __half2float(sh[gi]);
+          }
           int zq = 0;
           if (sc[gi] != 0.0f) {
             inv[gi] = __frcp_rn(sc[gi]);
@@ -904,7 +939,12 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
     if (valid) {
       reinterpret_cast<uint4*>(dcodes)[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
       reinterpret_cast<uint4*>(dcodes)[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-      if constexpr (ng == 4) {
+      if (L.sf) {
+        uint8_t* dsc = tb + (is_key ? L.k_scales : L.v_scales) + (int64_t)tid * ng;
+    #pragma unroll
+        for (int gi = 0; gi < ng; ++gi) dsc[gi] = (uint8_t)scode[gi];
+        reinterpret_cast<__half*>(tb + (is_key ? L.k_s2 : L.v_s2))[tid] = s2h;
+      } else if constexpr (ng == 4) {
         uint2 sv;
         sv.x = (uint32_t)__half_as_ushort(sh[0]) | ((uint32_t)__half_as_ushort(sh[1]) << 16);
         sv.y = (uint32_t)__half_as_ushort(sh[2]) | ((uint32_t)__half_as_ushort(sh[3]) << 16);

@@ -222,8 +222,31 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
       hi = fmaxf(hi, __shfl_xor_sync(0xFFFFFFFFu, hi, off));
     }
     const float s32 = __fdiv_rn(__fsub_rn(hi, lo), 3.0f);
-    const __half sh = __float2half_ru(s32);
-    const float sc = __half2float(sh);
+    __half sh = __float2half_ru(s32);
+    float sc = __half2float(sh);
+    // scale format 1 (App. D.1): s = code * s2, s2 the binary16 round-up of the
+    // token's largest range / 3 / 255, code the smallest byte covering range / 3
+    uint32_t code = 0;
+    __half s2h = __ushort_as_half(0);
+    if (L.sf) {
+      float smax = s32;
+      for (int off = glanes; off < 32; off <<= 1) smax = fmaxf(smax, __shfl_xor_sync(0xFFFFFFFFu, smax, off));
+      s2h = __float2half_ru(__fdiv_rn(smax, 255.0f));
+      float s2f = __half2float(s2h);
+      if (smax > 0.0f && __fmul_rn(255.0f, s2f) < smax) {
+        s2h = __ushort_as_half((unsigned short)(__half_as_ushort(s2h) + 1));
+        s2f = __half2float(s2h);
+      }
+      int c = 0;
+      if (s2f > 0.0f) {
+        c = (int)ceilf(__fdiv_rn(s32, s2f));
+        if (c > 0 && __fmul_rn((float)(c - 1), s2f) >= s32) c -= 1;
+        if (__fmul_rn((float)c, s2f) < s32) c += 1;
+        c = c > 255 ? 255 : c;
+      }
+      code = (uint32_t)c;
+      sc = __fmul_rn((float)c, s2f);
+    }
     int z = 0;
     uint32_t cbyte = 0;
     float k0[4];
@@ -262,8 +285,14 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
     word |= __shfl_xor_sync(0xFFFFFFFFu, word, 1);
     word |= __shfl_xor_sync(0xFFFFFFFFu, word, 2);
     if ((lane & 3) == 0) *reinterpret_cast<uint32_t*>(tb + o_codes + rowi * 32 + lane) = word;
-    if (lane % glanes == 0)
-      reinterpret_cast<__half*>(tb + o_scales + (int64_t)rowi * ng * 2)[lane / glanes] = sh;
+    if (lane % glanes == 0) {
+      if (L.sf) {
+        tb[o_scales + (int64_t)rowi * ng + lane / glanes] = (uint8_t)code;
+        if (lane == 0) reinterpret_cast<__half*>(tb + (is_key ? L.k_s2 : L.v_s2))[rowi] = s2h;
+      } else {
+        reinterpret_cast<__half*>(tb + o_scales + (int64_t)rowi * ng * 2)[lane / glanes] = sh;
+      }
+    }
     if (lane == 0) {
       tb[o_ids + rowi] = (uint8_t)id;
       tb[o_zeros + (int64_t)rowi * L.zb] = (uint8_t)zbyte;

@@ -182,6 +182,9 @@ __device__ __forceinline__ void qu_to_smem(uint8_t* sQU, int i, int row, uint32_
   }
 }
 
+// SF: the slot's scale format (0: binary16 group scales; 1: uint8 group codes
+// times a binary16 secondary scale per token, App. D.1).
+template <int SF>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     attend_kernel(const AttendArgs a, const AttendSlots S) {
   extern __shared__ uint8_t smem_raw[];
@@ -498,9 +501,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
               const uint8_t* cp = tb + L.k_codes + trw * 32;
               cwv[0] = __ldg(reinterpret_cast<const uint32_t*>(cp + 4 * q));
               cwv[1] = __ldg(reinterpret_cast<const uint32_t*>(cp + 16 + 4 * q));
-              const unsigned short* sp = reinterpret_cast<const unsigned short*>(tb + L.k_scales + (int64_t)trw * L.ng * 2);
-              scv[0] = __ldg(sp + ((16 * q) >> gshift));
-              scv[1] = __ldg(sp + ((64 + 16 * q) >> gshift));
+              if constexpr (SF == 0) {
+                const unsigned short* sp =
+                    reinterpret_cast<const unsigned short*>(tb + L.k_scales + (int64_t)trw * L.ng * 2);
+                scv[0] = __ldg(sp + ((16 * q) >> gshift));
+                scv[1] = __ldg(sp + ((64 + 16 * q) >> gshift));
+              } else {
+                const uint8_t* cp8 = tb + L.k_scales + (int64_t)trw * L.ng;
+                const __half s2 = __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(tb + L.k_s2) + trw));
+                scv[0] = __half_as_ushort(__hmul(__uint2half_rn(__ldg(cp8 + ((16 * q) >> gshift))), s2));
+                scv[1] = __half_as_ushort(__hmul(__uint2half_rn(__ldg(cp8 + ((64 + 16 * q) >> gshift))), s2));
+              }
               if (psac_lane) {
                 cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
                 sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
@@ -622,7 +633,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
               if (tb) {
                 ldg32B(tab + (int64_t)((idc >> (8 * p)) & 0xFFu) * 256 + 32 * c16, mv[pp]);
                 cwv[pp] = __ldg(reinterpret_cast<const uint32_t*>(tb + L.v_codes + row * 32 + 4 * c16));
-                scv[pp] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.v_scales + (int64_t)row * L.ng * 2) + g);
+                if constexpr (SF == 0) {
+                  scv[pp] = __ldg(reinterpret_cast<const unsigned short*>(tb + L.v_scales + (int64_t)row * L.ng * 2) + g);
+                } else {
+                  const __half s2 = __ushort_as_half(__ldg(reinterpret_cast<const unsigned short*>(tb + L.v_s2) + row));
+                  scv[pp] = __half_as_ushort(__hmul(__uint2half_rn(__ldg(tb + L.v_scales + (int64_t)row * L.ng + g)), s2));
+                }
               } else {
                 const __nv_bfloat16* src = a.vcur + ((size_t)(cur.tl * 128 + row) * H + h) * 128 + 16 * c16;
                 const uint4 f0 = bf16x8_to_f16x8(ldg16(src)), f1 = bf16x8_to_f16x8(ldg16(src + 8));
@@ -761,12 +777,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
 }  // namespace
 
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(attend_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  auto kern = a.L.sf ? attend_kernel<1> : attend_kernel<0>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
   // pairs of 256-query CTAs; an odd count gets one CTA with no queries
   const unsigned blocks = (unsigned)((a.Nq + 255) / 256);
   dim3 grid((blocks + 1) & ~1u, (unsigned)a.L.H);
-  attend_kernel<<<grid, NT, SMEM_BYTES, st>>>(a, slots);
+  kern<<<grid, NT, SMEM_BYTES, st>>>(a, slots);
   return cudaGetLastError();
 }
 

@@ -5,7 +5,8 @@
 //
 //   dequant_kernel  warp per (token, head), lane = four channels: the values
 //                   attention rebuilds, k_hat = mu_id + s (q - z) (+ U_r t sigma
-//                   for Keys stored with a PSAC correction), in fp32.
+//                   for Keys stored with a PSAC correction), in fp32; s is the
+//                   binary16 group scale or, in scale format 1, code * s2.
 //   top1_kernel     64 queries x 64 keys per step on CUDA cores (a measurement,
 //                   not the hot path): every logit is the fp32 sum in channel
 //                   order with one fused multiply-add per term; the largest
@@ -35,7 +36,9 @@ __global__ void __launch_bounds__(256) dequant_kernel(const DequantArgs a) {
     const int64_t o_ids = side ? L.v_ids : L.k_ids, o_zeros = side ? L.v_zeros : L.k_zeros;
     const int id = tb[o_ids + row];
     const __half* tab = reinterpret_cast<const __half*>(head + (side ? L.vtab : L.ktab)) + (size_t)id * 128;
-    const float s = __half2float(reinterpret_cast<const __half*>(tb + o_scales + row * ng * 2)[g]);
+    const float s = L.sf ? (float)tb[o_scales + row * ng + g] *
+                               __half2float(reinterpret_cast<const __half*>(tb + (side ? L.v_s2 : L.k_s2))[row])
+                         : __half2float(reinterpret_cast<const __half*>(tb + o_scales + row * ng * 2)[g]);
     const int z = (tb[o_zeros + row * L.zb + (g >> 2)] >> (2 * (g & 3))) & 3;
     const uint32_t word = reinterpret_cast<const uint32_t*>(tb + o_codes + row * 32)[c0 >> 4];
     const int m = (c0 & 15) >> 2;  // channels 4m .. 4m + 3 of the word's 16

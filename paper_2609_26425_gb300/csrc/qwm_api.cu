@@ -75,6 +75,7 @@ bool qwm::config_supported(const qwm_config* c) {
   if (c->num_centroids < 1 || c->num_centroids > 256) return false;
   if (c->psac_rank != 0 && c->psac_rank != 8 && c->psac_rank != 16 && c->psac_rank != 32) return false;
   if (c->num_candidates < 1 || c->kmeans_iters < 0) return false;
+  if (c->scale_format != 0 && c->scale_format != 1) return false;
   return true;
 }
 
@@ -82,7 +83,7 @@ namespace {
 
 bool same_shape(const qwm_config* a, const qwm_config* b) {
   return a->num_heads == b->num_heads && a->head_dim == b->head_dim && a->num_centroids == b->num_centroids &&
-         a->group_size == b->group_size && a->psac_rank == b->psac_rank;
+         a->group_size == b->group_size && a->psac_rank == b->psac_rank && a->scale_format == b->scale_format;
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -193,6 +194,8 @@ qwm_status qwm_cache_layout(const qwm_cache* c, qwm_layout* o) {
   o->v_codes = L.v_codes; o->v_scales = L.v_scales; o->v_ids = L.v_ids; o->v_zeros = L.v_zeros;
   o->v_bytes = L.v_bytes;
   o->zero_bytes = L.zb;
+  o->k_s2 = L.k_s2;
+  o->v_s2 = L.v_s2;
   return QWM_OK;
 }
 

@@ -24,11 +24,13 @@ __host__ __device__ inline int64_t round_up(int64_t x, int64_t a) { return (x + 
 // Byte layout of the packed cache (see qwm_layout in qwm.h).
 struct Layout {
   int H, d, C, G, r, ng, zb;
+  int sf;                // scale format: 0 binary16 scales, 1 uint8 codes + binary16 secondary scale
   int64_t T;             // token capacity of a slot
   int32_t max_chunks;
   int64_t tiles;         // tiles per slot
   int64_t k_codes, k_scales, k_ids, k_zeros, k_coef, k_sigma, k_bytes;
   int64_t v_codes, v_scales, v_ids, v_zeros, v_bytes;  // from the tile start
+  int64_t k_s2, v_s2;    // scale format 1: secondary scales [128] binary16
   int64_t tile_bytes;
   int64_t ktab, vtab, ut, tiles_off, head_bytes;
   int64_t slot_bytes;
@@ -38,13 +40,15 @@ struct Layout {
 inline Layout make_layout(const qwm_config& c, int64_t T, int32_t max_chunks) {
   Layout L{};
   L.H = c.num_heads; L.d = c.head_dim; L.C = c.num_centroids; L.G = c.group_size; L.r = c.psac_rank;
+  L.sf = c.scale_format;
   L.ng = L.d / L.G;
   L.zb = (2 * L.ng + 7) / 8;
   L.T = T; L.max_chunks = max_chunks;
   L.tiles = (T + kTile - 1) / kTile;
   int64_t o = 0;
   L.k_codes = o;  o += (int64_t)kTile * (L.d / 4);
-  L.k_scales = o; o += round_up((int64_t)kTile * L.ng * 2, 16);
+  L.k_scales = o; o += round_up((int64_t)kTile * L.ng * (L.sf ? 1 : 2), 16);
+  L.k_s2 = L.sf ? o : 0; o += L.sf ? kTile * 2 : 0;
   L.k_ids = o;    o += kTile;
   L.k_zeros = o;  o += round_up((int64_t)kTile * L.zb, 16);
   L.k_coef = o;   o += (int64_t)kTile * L.r;
@@ -52,7 +56,8 @@ inline Layout make_layout(const qwm_config& c, int64_t T, int32_t max_chunks) {
   L.k_bytes = round_up(o, 128);
   o = L.k_bytes;
   L.v_codes = o;  o += (int64_t)kTile * (L.d / 4);
-  L.v_scales = o; o += round_up((int64_t)kTile * L.ng * 2, 16);
+  L.v_scales = o; o += round_up((int64_t)kTile * L.ng * (L.sf ? 1 : 2), 16);
+  L.v_s2 = L.sf ? o : 0; o += L.sf ? kTile * 2 : 0;
   L.v_ids = o;    o += kTile;
   L.v_zeros = o;  o += round_up((int64_t)kTile * L.zb, 16);
   L.v_bytes = round_up(o, 128) - L.k_bytes;

@@ -24,16 +24,20 @@ ATT_MAX_ABS = 2e-2
 ATT_MEAN_ABS = 2e-3
 
 
-def oracle_append(k_bits, v_bits, kc_bits, vc_bits, *, G, r, M, w=None, U_bits=None, nthreads=0):
+def oracle_append(k_bits, v_bits, kc_bits, vc_bits, *, G, r, M, w=None, U_bits=None, nthreads=0,
+                  two_level=False):
     """Oracle packed Keys and Values of one chunk (token-major dicts)."""
-    ko = orc.quantize(k_bits, kc_bits, G=G, r=r, M=M, is_key=True, w=w, U_bits=U_bits, nthreads=nthreads)
-    vo = orc.quantize(v_bits, vc_bits, G=G, r=r, M=M, is_key=False, nthreads=nthreads)
+    ko = orc.quantize(k_bits, kc_bits, G=G, r=r, M=M, is_key=True, w=w, U_bits=U_bits, nthreads=nthreads,
+                      two_level_scales=two_level)
+    vo = orc.quantize(v_bits, vc_bits, G=G, r=r, M=M, is_key=False, nthreads=nthreads, two_level_scales=two_level)
     return ko, vo
 
 
 def compare_packed(gpu: dict, ref: dict, x_bits, cent_bits, *, G, r, M, is_key, w=None, U_bits=None,
-                   prefix=""):
-    """Assert bit-exact parity of one side (Keys: prefix '', Values: prefix 'v_')."""
+                   prefix="", two_level=False):
+    """Assert bit-exact parity of one side (Keys: prefix '', Values: prefix 'v_').
+    two_level: the slot stores uint8 group codes and a binary16 secondary scale
+    (scale format 1) instead of binary16 group scales."""
     g_ids = gpu[prefix + "ids"]
     diff = g_ids != ref["ids"]
     stats = {"tokens": int(g_ids.size), "id_flips": int(diff.sum())}
@@ -42,8 +46,8 @@ def compare_packed(gpu: dict, ref: dict, x_bits, cent_bits, *, G, r, M, is_key, 
         bad = diff & (margin >= ID_MARGIN)
         assert not bad.any(), f"{int(bad.sum())} id mismatches with oracle margin >= {ID_MARGIN}"
         ref = orc.quantize(x_bits, cent_bits, G=G, r=r, M=M, is_key=is_key, w=w, U_bits=U_bits,
-                           force_ids=g_ids)
-    for key in ("codes", "zeros", "scales"):
+                           force_ids=g_ids, two_level_scales=two_level)
+    for key in ("codes", "zeros") + (("scode", "s2") if two_level else ("scales",)):
         a, b = gpu[prefix + key], ref[key]
         assert a.shape == b.shape, (key, a.shape, b.shape)
         nbad = int((a != b).sum())

@@ -57,7 +57,7 @@ def make_chunk(seed, N, H, *, outliers=True):
     return q, k, v
 
 
-def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None):
+def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None, scale_format=0):
     _, k, v = make_chunk(seed, N, H)
     kb, vb = synth.bits(k), synth.bits(v)
     if fit_iters:
@@ -67,17 +67,18 @@ def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None
         kc, vc = strided_centroids(kb, C), strided_centroids(vb, C)
     w = synth.random_weights(seed + 100, H, 128).numpy() if use_w else None
     Ub = synth.bits(synth.random_orthonormal(seed + 200, H, 128, r)) if (use_U and r > 0) else None
-    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, scale_format=scale_format)
     cache = qwm.Cache(cfg, T or N, 2)
+    tl = scale_format == 1
     qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
                             w=None if w is None else torch.from_numpy(w).cuda(),
                             U=None if Ub is None else dev(synth.from_bits(Ub)))
     torch.cuda.synchronize()
     assert cache.status() == 0
     dec = cache.decode_chunk(0)
-    ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub)
-    sk = compare_packed(dec, ko, kb, kc, G=G, r=r, M=M, is_key=True, w=w, U_bits=Ub)
-    sv = compare_packed(dec, vo, vb, vc, G=G, r=r, M=M, is_key=False, prefix="v_")
+    ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub, two_level=tl)
+    sk = compare_packed(dec, ko, kb, kc, G=G, r=r, M=M, is_key=True, w=w, U_bits=Ub, two_level=tl)
+    sv = compare_packed(dec, vo, vb, vc, G=G, r=r, M=M, is_key=False, prefix="v_", two_level=tl)
     assert np.array_equal(dec["k_tab"], f16_bits(kc)) and np.array_equal(dec["v_tab"], f16_bits(vc))
     if Ub is not None:
         assert np.array_equal(dec["U"], Ub)
@@ -97,6 +98,19 @@ def run_append_case(H, N, C, G, r, M, use_w, use_U, seed, fit_iters=None, T=None
 ])
 def test_append_parity(H, N, C, G, r, M, use_w, use_U):
     sk, sv = run_append_case(H, N, C, G, r, M, use_w, use_U, seed=H * 1000 + N)
+    assert sk["id_flips"] <= max(1, N * H // 1000)
+
+
+@pytest.mark.parametrize("H,N,C,G,r,M", [
+    (4, 880, 64, 32, 16, 4),      # the single-layer workload's shape
+    (2, 300, 256, 64, 32, 2),     # G = 64
+    (2, 150, 64, 32, 16, 12),     # 8 < M < C: the generic kernel
+    (1, 1, 4, 32, 8, 4),          # a single token
+])
+def test_append_parity_two_level_scales(H, N, C, G, r, M):
+    """Scale format 1 (App. D.1): uint8 group codes with a binary16 secondary
+    scale per token-head, bit-exact against the oracle's two-level scales."""
+    sk, sv = run_append_case(H, N, C, G, r, M, True, True, seed=H * 1000 + N + 7, scale_format=1)
     assert sk["id_flips"] <= max(1, N * H // 1000)
 
 
@@ -158,9 +172,9 @@ def test_fit_parity_full_size_sampled():
 
 
 def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, window=0, max_chunks=None,
-                              psac_chunks=None, rows=None):
+                              psac_chunks=None, rows=None, scale_format=0):
     """Append chunks on the GPU and build the oracle's reference keys/values."""
-    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, scale_format=scale_format)
     T = max(chunk_sizes)
     cache = qwm.Cache(cfg, T, max_chunks or len(chunk_sizes), sliding_window=bool(window))
     Ks, Vs = [], []
@@ -174,7 +188,7 @@ def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, win
         qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
                                 w=None if w is None else torch.from_numpy(w).cuda(),
                                 U=None if Ub is None else dev(synth.from_bits(Ub)))
-        ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub)
+        ko, vo = oracle_append(kb, vb, kc, vc, G=G, r=r, M=M, w=w, U_bits=Ub, two_level=scale_format == 1)
         K, V = oracle_kv(ko, vo, kc, vc, G=G, r=r, U_bits=Ub)
         Ks.append(K)
         Vs.append(V)
@@ -202,6 +216,24 @@ def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, win
 def test_attend_parity(H, chunks, C, G, r, Ncur, Nq):
     cfg, cache, q, kc, vc, ref, lse = build_cache_and_reference(H, chunks, C, G, r, 4, seed=31 * H + Nq,
                                                                Ncur=Ncur, Nq=Nq)
+    out, lse_g = qwm.qwm_attend(cfg, cache, dev(q), dev(kc) if Ncur else None, dev(vc) if Ncur else None,
+                                want_lse=True)
+    torch.cuda.synchronize()
+    assert cache.status() == 0
+    compare_attention(out.float().cpu().numpy(), ref)
+    assert np.abs(lse_g.cpu().numpy() - lse).max() < 2e-2
+
+
+@pytest.mark.parametrize("H,chunks,C,G,r,Ncur,Nq", [
+    (4, [880, 880], 64, 32, 16, 880, 880),
+    (2, [300, 77], 16, 64, 8, 129, 200),
+])
+def test_attend_parity_two_level_scales(H, chunks, C, G, r, Ncur, Nq):
+    """Attention over a cache stored with scale format 1 (group scale = code *
+    secondary scale, rebuilt in binary16) against the oracle's fp64 attention
+    over its own two-level reconstruction."""
+    cfg, cache, q, kc, vc, ref, lse = build_cache_and_reference(H, chunks, C, G, r, 4, seed=37 * H + Nq,
+                                                               Ncur=Ncur, Nq=Nq, scale_format=1)
     out, lse_g = qwm.qwm_attend(cfg, cache, dev(q), dev(kc) if Ncur else None, dev(vc) if Ncur else None,
                                 want_lse=True)
     torch.cuda.synchronize()
