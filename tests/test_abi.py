@@ -104,3 +104,21 @@ def test_query_statistics_and_measurement_host_errors(qlib):
     assert L.qwm_top1_keys(ct.byref(bad), fake, 10, fake, 10, fake, None) == 2
     assert L.qwm_top1_keys(ct.byref(cfg), fake, 10, ct.c_void_p((1 << 20) + 4), 10, fake, None) == 1
     assert L.qwm_dequant_chunk(ct.byref(cfg), None, 0, fake, None, None) == 1
+
+
+def test_cache_bytes_two_level_scales(qlib):
+    """Scale format 1 (App. D.1): per token-head d/G uint8 scale codes and one
+    binary16 secondary scale replace the d/G binary16 scales, for Keys and
+    Values alike (58 + 40 bytes instead of 60 + 42 at G = 32, r = 16)."""
+    for (H, C, G, r, T, n) in [(40, 256, 32, 16, 4680, 6), (4, 64, 64, 8, 880, 3), (2, 16, 32, 0, 100, 1)]:
+        cfg = qlib.config(H, C, group_size=G, psac_rank=r, scale_format=1)
+        b = qlib.qwm_cache_bytes(cfg, T, n)
+        d, ng = 128, 128 // G
+        k_tok = d // 4 + ng + 2 + 1 + 1 + (r + 2 if r else 0)
+        v_tok = d // 4 + ng + 2 + 1 + 1
+        tiles = -(-T // 128)
+        per_head = 2 * C * d * 2 + r * d * 2
+        per_head = -(-per_head // 1024) * 1024 + tiles * 128 * (k_tok + v_tok)
+        per_head = -(-per_head // 1024) * 1024
+        assert b == 256 + n * (256 + H * per_head)
+    assert qlib.qwm_cache_bytes(qlib.config(4, 64, scale_format=2), 100, 2) == 0
