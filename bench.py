@@ -35,15 +35,16 @@ METRIC = "attend TFLOP/s + append GB/s per chunk, GB300 roofline % (1 GPU)"
 UNIT = "TFLOP/s"
 
 
-def workload_numbers(wl):
+def workload_numbers(wl, scale_format=0):
     """Algorithmic work of one step (one layer-chunk)."""
     H, d, N, C, G, r = wl.heads, wl.head_dim, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank
     L = wl.cache_tokens
     Nq = Ncur = N
     attend_flops = 2.0 * H * Nq * (L * (2 * d + r) + Ncur * 2 * d)
     ng = d // G
-    k_tok = d // 4 + 2 * ng + 1 + 1 + (r + 2 if r else 0)
-    v_tok = d // 4 + 2 * ng + 1 + 1
+    scale_b = ng + 2 if scale_format else 2 * ng   # uint8 codes + binary16 secondary, or binary16 per group
+    k_tok = d // 4 + scale_b + 1 + 1 + (r + 2 if r else 0)
+    v_tok = d // 4 + scale_b + 1 + 1
     reads = 2 * N * H * d * 2 + 2 * H * C * d * 2 + H * d * r * 2 + H * d * 4
     writes = N * H * (k_tok + v_tok) + 2 * H * C * d * 2 + H * r * d * 2
     return {"attend_flops": attend_flops, "append_bytes": float(reads + writes),
@@ -169,7 +170,8 @@ def run_gpu(args, wl, rank, world):
     dev = torch.device("cuda", local)
     qwm.lib()
     H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
-    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, kmeans_iters=wl.kmeans_iters)
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, kmeans_iters=wl.kmeans_iters,
+                     scale_format=args.scale_format)
     src = synth.ChunkSource(wl, layer=rank)
     ws = torch.empty(qwm.qwm_fit_workspace_bytes(cfg, N), dtype=torch.uint8, device=dev)
 
@@ -203,7 +205,7 @@ def run_gpu(args, wl, rank, world):
     out = torch.empty_like(qd)
     torch.cuda.synchronize()
 
-    nums = workload_numbers(wl)
+    nums = workload_numbers(wl, args.scale_format)
     stream = torch.cuda.current_stream()
 
     def step(ev=None):
@@ -323,6 +325,8 @@ def run_gpu(args, wl, rank, world):
         "config": {"workload": wl.name, "heads": H, "head_dim": wl.head_dim, "chunk_tokens": N,
                    "cached_tokens": wl.cache_tokens, "active_tokens": N, "query_tokens": N,
                    "centroids": C, "group_size": G, "psac_rank": r, "candidates": M,
+                   "scale_format": "binary16 group scales" if args.scale_format == 0 else
+                   "uint8 group codes x binary16 secondary scale",
                    "parallelism": f"replicas{world}" if world > 1 else "single",
                    "l2": "inputs larger than L2 (packed history %.0f MB + q/k/v %.0f MB per step)" % (
                        hist.nbytes / 1e6, 3 * qd.numel() * 2 / 1e6)},
@@ -364,13 +368,14 @@ def top1_shift_measure(qwm, wl, hist, past, qd, dev, every=9):
     import torch
     H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
     qs = qd[::every].contiguous()
-    cfg_ref = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M)
+    sf = hist.cfg.scale_format
+    cfg_ref = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, scale_format=sf)
     k_ref = torch.cat([p[0].float() for p in past])
     idx_ref = qwm.qwm_top1_keys(cfg_ref, qs, k_ref)
     del k_ref
     out = {}
-    variants = (("qvg", qwm.config(H, C, group_size=G, psac_rank=0, candidates=1), False, False),
-                ("qsac", qwm.config(H, C, group_size=G, psac_rank=0, candidates=M), True, False),
+    variants = (("qvg", qwm.config(H, C, group_size=G, psac_rank=0, candidates=1, scale_format=sf), False, False),
+                ("qsac", qwm.config(H, C, group_size=G, psac_rank=0, candidates=M, scale_format=sf), True, False),
                 ("qsac_psac", cfg_ref, True, True))
     for name, cfg, use_w, use_U in variants:
         if name == "qsac_psac":
@@ -524,7 +529,7 @@ def run_reference(args, wl):
     for _ in range(args.steps):
         full, desc, _ = oracle_sample(wl, 128, 8, 2, nthreads)
         times.append(full)
-    nums = workload_numbers(wl)
+    nums = workload_numbers(wl, args.scale_format)
     sec = sum(times) / len(times)
     value = nums["attend_flops"] / sec / 1e12
     return {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "impl": "reference", "n_gpus": 0,
@@ -546,6 +551,8 @@ def main():
     ap.add_argument("--workload", default="wan14b_layer")
     ap.add_argument("--cpu-threads", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--scale-format", type=int, default=0, choices=[0, 1],
+                    help="group scale storage: 0 binary16 per group, 1 uint8 codes + binary16 per token")
     ap.add_argument("--heads", type=int, default=0,
                     help="profiling only: the workload with fewer heads (same per-head work); not a bench line")
     args = ap.parse_args()
