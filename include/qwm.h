@@ -80,15 +80,21 @@ typedef struct qwm_cache qwm_cache;
 
 /* Byte offsets of the packed cache, for readers of the buffer (tests, tools).
  * A slot holds one chunk: for head h, at slot_offset(s) + slot_meta_bytes +
- * h*head_bytes, come the Key centroid table [C][d] bf16, the Value centroid
- * table [C][d] bf16, U_r^T [r][d] bf16, then tiles_per_chunk tiles of
- * tile_tokens tokens.  Each tile is a Key block followed by a Value block of
- * structure-of-arrays fields (offsets within the tile): codes [128][d/4] u8
- * (channel c in byte c/4, bits 2(c%4)), scales [128][d/G] binary16,
- * ids [128] u8, zero-points [128][zb] u8 (group g in byte g/4, bits 2(g%4)),
- * and for Keys PSAC codes [128][r] int8 and row scales [128] binary16.  With
- * scale_format 1 the scale field holds [128][d/G] u8 codes and a secondary
- * scale field [128] binary16 follows it (k_s2, v_s2). */
+ * h*head_bytes, come the Key centroid table [C][d] and the Value centroid
+ * table [C][d], both binary16 (the chunk's bf16 tables converted exactly;
+ * bf16 values outside the binary16 range are not representable there),
+ * U_r^T [r][d] bf16, then tiles_per_chunk tiles of tile_tokens tokens.  Each
+ * tile is a Key block followed by a Value block of structure-of-arrays fields
+ * (offsets within the tile):
+ *   codes [128][d/4] u8: the 2-bit codes of a token, 16 channels per
+ *     little-endian 32-bit word; in word k (channels 16k..16k+15) the even
+ *     channel 16k+2i sits at bits 2i and the odd channel 16k+2i+1 at bits
+ *     16+2i (App. D.1 packs four codes per byte; this order is ours);
+ *   scales [128][d/G] binary16; ids [128] u8;
+ *   zero-points [128][zb] u8: group g in byte g/4, bits 2(g%4);
+ *   Keys only: PSAC codes [128][r] int8 and row scales [128] binary16.
+ * With scale_format 1 the scale field holds [128][d/G] u8 codes and a
+ * secondary scale field [128] binary16 follows it (k_s2, v_s2). */
 typedef struct qwm_layout {
   int64_t header_bytes;     /* device status word + reserved, before slot 0 */
   int64_t slot_meta_bytes;  /* per-slot reserved bytes before head 0 */
@@ -109,8 +115,9 @@ QWM_API const char* qwm_status_string(qwm_status status);
 /* Bytes of device memory a cache of max_chunks slots of tokens_per_chunk
  * tokens needs (App. D.1 packed storage: per token-head d/4 code bytes, d/G
  * binary16 scales, one uint8 centroid id, 2-bit zero-points, for Keys r INT8
- * PSAC codes + one binary16 row scale; per chunk-head the two bf16 centroid
- * tables and U_r).  Returns 0 for an invalid or unsupported configuration. */
+ * PSAC codes + one binary16 row scale; per chunk-head the two centroid
+ * tables as binary16 and U_r^T as bf16).  Returns 0 for an invalid or
+ * unsupported configuration. */
 QWM_API size_t qwm_cache_bytes(const qwm_config* cfg, int64_t tokens_per_chunk, int32_t max_chunks);
 
 /* Create a host descriptor over dev_buf (256-byte aligned, bytes >=

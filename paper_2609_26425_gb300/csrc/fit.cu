@@ -678,13 +678,6 @@ constexpr int kMaxDevices = 64;
 std::mutex g_fit_scratch_mutex;
 void* g_fit_scratch_addr[kMaxDevices] = {};
 
-bool noalloc_cfg_ok(const qwm_config* c) {
-  return c->num_heads >= 1 && c->num_heads <= 4096 && c->head_dim == kHeadDim &&
-         (c->group_size == 32 || c->group_size == 64) && c->num_centroids >= 1 && c->num_centroids <= 256 &&
-         (c->psac_rank == 0 || c->psac_rank == 8 || c->psac_rank == 16 || c->psac_rank == 32) &&
-         c->num_candidates >= 1 && c->kmeans_iters >= 0;
-}
-
 }  // namespace
 }  // namespace qwm
 
@@ -692,7 +685,7 @@ extern "C" QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, c
                                                         void* centroids, void* stream) {
   using namespace qwm;
   if (!cfg || !x || !centroids || N < 1) return QWM_ERR_INVALID_ARG;
-  if (!noalloc_cfg_ok(cfg)) return QWM_ERR_UNSUPPORTED;
+  if (!config_supported(cfg)) return QWM_ERR_UNSUPPORTED;  // the same set qwm_fit_centroids accepts
   if (N > (int64_t)1 << 31) return QWM_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(x) & 15u) || (reinterpret_cast<uintptr_t>(centroids) & 15u))
     return QWM_ERR_INVALID_ARG;

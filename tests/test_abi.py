@@ -122,3 +122,19 @@ def test_cache_bytes_two_level_scales(qlib):
         per_head = -(-per_head // 1024) * 1024
         assert b == 256 + n * (256 + H * per_head)
     assert qlib.qwm_cache_bytes(qlib.config(4, 64, scale_format=2), 100, 2) == 0
+
+
+def test_fit_entry_points_accept_the_same_configurations(qlib):
+    """The allocation-free k-means entry point rejects exactly what the
+    workspace entry point rejects (an unsupported scale format, rank or
+    group size) before anything reaches CUDA."""
+    L = qlib.lib()
+    fn = L.qwm_fit_centroids_noalloc
+    fn.argtypes = [ct.c_void_p, ct.c_void_p, ct.c_int64, ct.c_void_p, ct.c_void_p]
+    fn.restype = ct.c_int
+    fake = ct.c_void_p(1 << 20)
+    for bad in (qlib.config(4, 64, scale_format=2), qlib.config(4, 64, psac_rank=12),
+                qlib.config(4, 64, group_size=16), qlib.config(4, 300)):
+        assert L.qwm_fit_centroids(ct.byref(bad), fake, 10, fake, fake, 1 << 30, None) == 2
+        assert fn(ct.byref(bad), fake, 10, fake, None) == 2
+    assert fn(ct.byref(qlib.config(4, 64)), fake, 0, fake, None) == 1

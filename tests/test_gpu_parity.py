@@ -157,6 +157,23 @@ def test_fit_parity_off_grid_members():
     assert np.array_equal(got, ref["centroids"])
 
 
+@pytest.mark.parametrize("rows,C,iters", [
+    ([(2.0, 0.0), (-2.0, 0.0), (0.0, 1.0)], 2, 1),                 # exact tie -> lower index
+    ([(1.0, 0.0), (1.0, 0.5), (1.0, 0.0), (1.0, 1.5)], 2, 1),      # cluster 1 empty after step 1
+    ([(1.0, 0.0), (1.0, 0.5), (1.0, 0.0), (1.0, 1.5)], 2, 2),
+])
+def test_fit_parity_ties_and_empty_clusters(rows, C, iters):
+    """The hand fixtures of the oracle's k-means pins (exact distance ties,
+    an empty cluster keeping its centroid) give the same centroids on the GPU."""
+    x = np.zeros((len(rows), 1, 128), np.float32)
+    for i, row in enumerate(rows):
+        x[i, 0, : len(row)] = row
+    xt = torch.from_numpy(x).to(torch.bfloat16)
+    ref = orc.fit_centroids(synth.bits(xt), C, iters)
+    got = synth.bits(qwm.qwm_fit_centroids(qwm.config(1, C, kmeans_iters=iters), dev(xt)).cpu())
+    assert np.array_equal(got, ref["centroids"])
+
+
 def test_fit_parity_full_size_sampled():
     """The Wan-14B-shaped Keys and Values (40 heads, 4680 tokens, 256
     centroids, 10 iterations); the oracle runs on three sampled heads."""

@@ -89,6 +89,53 @@ def test_fit_init_is_strided_tokens(orc):
     assert np.array_equal(o["centroids"][0], x[idx, 0])
 
 
+def tokens(rows, d=128):
+    """bf16 bits [N][1][d] of tokens given by their first channels."""
+    x = np.zeros((len(rows), 1, d), np.float32)
+    for i, row in enumerate(rows):
+        x[i, 0, : len(row)] = row
+    return synth.bits(torch.from_numpy(x).to(torch.bfloat16))
+
+
+def first_channels(bits, n):
+    return orc_f32(bits)[..., :n]
+
+
+def orc_f32(bits):
+    return (np.asarray(bits, np.uint32) << 16).view(np.float32)
+
+
+def test_fit_tie_goes_to_lower_index(orc):
+    """A token at exactly the same distance from two centroids joins the one
+    with the lower index (the assignment convention of k-means in Sec. 2).
+    Tokens (2, 0), (-2, 0), (0, 1); initial centroids are tokens 0 and 1
+    (token floor(j N / C)); token 2 is at distance 5 from both, so it joins
+    cluster 0: after one step the centroids are (1, 0.5) and (-2, 0) -- the
+    other choice would give (2, 0) and (-1, 0.5)."""
+    x = tokens([(2.0, 0.0), (-2.0, 0.0), (0.0, 1.0)])
+    o = orc.fit_centroids(x, C=2, iters=1)
+    c = first_channels(o["centroids"][0], 3)
+    assert np.array_equal(c, np.array([[1.0, 0.5, 0.0], [-2.0, 0.0, 0.0]], np.float32))
+    assert not orc_f32(o["centroids"][0])[:, 3:].any()
+    assert list(o["assign"][:, 0]) == [0, 1, 0]
+
+
+def test_fit_empty_cluster_keeps_its_centroid(orc):
+    """An empty cluster keeps its previous centroid (Sec. 2 k-means; Lloyd's
+    update has no mean for it).  Tokens (1, 0), (1, 0.5), (1, 0), (1, 1.5);
+    the initial centroids are tokens 0 and 2, which are equal, so every token
+    is equally far from both and joins cluster 0 (lower index): cluster 1 is
+    empty after the first step and stays at (1, 0) while cluster 0 moves to
+    the mean (1, 0.5).  The second step splits the tokens: (1, 0) and (1, 0)
+    go to cluster 1, the others to cluster 0, whose mean is (1, 1)."""
+    x = tokens([(1.0, 0.0), (1.0, 0.5), (1.0, 0.0), (1.0, 1.5)])
+    o1 = orc.fit_centroids(x, C=2, iters=1)
+    assert np.array_equal(first_channels(o1["centroids"][0], 2), np.array([[1.0, 0.5], [1.0, 0.0]], np.float32))
+    o2 = orc.fit_centroids(x, C=2, iters=2)
+    assert np.array_equal(first_channels(o2["centroids"][0], 2), np.array([[1.0, 1.0], [1.0, 0.0]], np.float32))
+    assert list(o2["assign"][:, 0]) == [1, 0, 1, 0]
+
+
 def test_fit_matches_sklearn_lloyd(orc):
     sk = pytest.importorskip("sklearn.cluster")
     N, H, d, C, iters = 800, 1, 128, 12, 6

@@ -59,6 +59,18 @@ MUTATIONS = [
      'M = np.einsum("nhc,nhe->hce", q, q) / N',
      'M = np.einsum("nhc,nhe->hce", q, q) / max(N - 1, 1)',
      [(pins_af.test_query_stats_hadamard_closed_form, {}), (pins_af.test_query_stats_diagonal_weights, {})]),
+    ("PSAC INT8 codes truncated instead of rounded", "qwm_oracle.c",
+     "float qq = rint_even(y);",
+     "float qq = truncf(y);",
+     [(pins_q.test_psac_int8_rounding_hand_fixture, {})]),
+    ("k-means tie goes to the higher index", "qwm_oracle.c",
+     "if (bj < 0 || acc < best) { best = acc; bj = j; }\n        }\n        lab[i] = bj;",
+     "if (bj < 0 || acc <= best) { best = acc; bj = j; }\n        }\n        lab[i] = bj;",
+     [(pins_af.test_fit_tie_goes_to_lower_index, {})]),
+    ("k-means empty cluster reset to zero", "qwm_oracle.c",
+     "if (cnt[j] == 0) continue;",
+     "if (cnt[j] == 0) { for (int c = 0; c < d; ++c) mu[(size_t)j * d + c] = 0.0f; continue; }",
+     [(pins_af.test_fit_empty_cluster_keeps_its_centroid, {})]),
     ("top-1 key by the smallest logit", "oracle.py",
      "idx[h] = np.argmax(L, axis=1)",
      "idx[h] = np.argmin(L, axis=1)",

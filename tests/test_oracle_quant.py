@@ -299,6 +299,44 @@ def test_psac_exact_when_error_in_span(orc):
         assert np.abs(o["coef"][i, 0]).max() == 127
 
 
+def psac_hand_token(g):
+    """The Key token, centroid and basis of the hand-computed INT8 fixture."""
+    d, G, r, s = g["head_dim"], g["group_size"], g["psac_rank"], g["grid_scale"]
+    m = ((7 * np.arange(d)) % 4 - 1).astype(np.float64)
+    m[::G] = -1
+    m[1::G] = 2
+    x = m * s
+    chans = np.array(g["target_channels"])
+    assert np.all(chans % G > 1), "target channels must not carry a group's range"
+    x[chans] = np.array(g["e_in_units_of_2^-10"]) * 2.0 ** -10
+    U = np.zeros((1, d, r), np.float32)
+    U[0, chans, np.arange(r)] = 1.0
+    return bf(x.reshape(1, 1, d)), np.zeros((1, 1, d), np.uint16), bf(U), chans
+
+
+def test_psac_int8_rounding_hand_fixture(orc):
+    """INT8 PSAC codes round half to even and sigma is the binary16 round-up of
+    max|c| / 127 (Sec. 4.2 Eq. 16, App. D.1; tests/golden/psac_int8_hand.json).
+    The coefficients land on exact halves, quarters and near-integers, so
+    truncation, rounding half away from zero, or a scale off by one binary16
+    step give different codes."""
+    g = json.load(open(os.path.join(GOLDEN, "psac_int8_hand.json")))
+    d, G, r = g["head_dim"], g["group_size"], g["psac_rank"]
+    x, cent, Ub, chans = psac_hand_token(g)
+    o = orc.quantize(x, cent, G=G, r=r, M=1, is_key=True, U_bits=Ub)
+    assert int(o["kept"][0, 0]) == 1
+    assert int(o["sigma"][0, 0]) == g["sigma_f16_bits"]
+    assert list(o["coef"][0, 0].astype(int)) == g["codes"]
+    # the grid channels reconstruct exactly, the targets carry only the correction
+    deq = orc.dequant(o, cent, G=G, r=r, U_bits=Ub)
+    want = orc.bf16_to_f32(x)[0, 0].astype(np.float64)
+    want[chans] = np.array(g["codes"]) * 2.0 ** -10
+    assert np.array_equal(deq[0, 0], want)
+    # with w = 1 and no correction stored, the zero codes are what a dropped row gives
+    o0 = orc.quantize(x, cent, G=G, r=0, M=1, is_key=True)
+    assert np.array_equal(o0["codes"], o["codes"]) and np.array_equal(o0["scales"], o["scales"])
+
+
 def test_psac_off_and_rank_zero(orc):
     N, H, d, C, G = 40, 2, 128, 16, 32
     x = synth.bits(synth.gaussian_bf16(71, N, H, d))
