@@ -106,6 +106,9 @@ constexpr int F_LIST = F_RED + 64;          // FNT x 32-byte records
 constexpr int F_BAR = F_LIST + FNT * 32;    // 4 mbarriers, flags, TMEM slot
 constexpr int F_SMEM = F_BAR + 64 + 1024;
 
+// CAPT = M + 1 (the ranked list of a row), or kMaxFilterM + 1 for the
+// candidate counts without their own instance.
+template <int CAPT>
 __global__ void __launch_bounds__(FNT, 1)
     append_filter(const AppendArgs a, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, int tiles, int units) {
@@ -279,76 +282,93 @@ __global__ void __launch_bounds__(FNT, 1)
       //   1. the minima of 16 interleaved column groups (column j in group
       //      j % 16); their (M+1)-th smallest, T, bounds the (M+1)-th
       //      smallest dt from above;
-      //   2. the few columns with dt <= T go, in ascending j, to a per-row
-      //      list in this group's A tile (free once the MMA has completed);
-      //   3. the M+1 smallest of the list are the M+1 smallest of the row.
-      constexpr int CAP = kMaxFilterM + 1;
-      constexpr int kList = 32;
-      const int nchunk = (Npad + 31) >> 5;
-      auto load_dt = [&](int cb, float (&v)[32]) {
-        __syncwarp();
-        tmem_ld32(tD + lrow + cb * 32, v);
+      //   2. a second pass marks the columns with dt <= T in a bit mask per
+      //      32 columns (usually a handful per row); only those are ranked
+      //      (the M+1 smallest, ties to the lower j) and listed, in
+      //      ascending j, in this group's A tile (free once the MMA has
+      //      completed), with the values of a 32-column block stashed there
+      //      when the block has one.
+      constexpr int kList = 16;
+      const int nchunk = ((Npad + 63) >> 6) << 1;  // pairs of 32-column blocks (at most 256 columns)
+      // dt of 32 consecutive columns from their D values, two at a time with
+      // packed fused multiply-adds (each lane rounds once, as fmaf(-2, D, A))
+      auto dt32 = [&](int cb, float (&v)[32]) {
         const float4* aj4 = reinterpret_cast<const float4*>(sAj + cb * 32);
+        const uint64_t M2 = f2pack(-2.0f, -2.0f);
 #pragma unroll
         for (int e = 0; e < 32; e += 4) {
           const float4 A4 = aj4[e >> 2];
-          v[e] = fmaf(-2.0f, v[e], A4.x);
-          v[e + 1] = fmaf(-2.0f, v[e + 1], A4.y);
-          v[e + 2] = fmaf(-2.0f, v[e + 2], A4.z);
-          v[e + 3] = fmaf(-2.0f, v[e + 3], A4.w);
+          const uint64_t r0 = fma2(f2pack(v[e], v[e + 1]), M2, f2pack(A4.x, A4.y));
+          const uint64_t r1 = fma2(f2pack(v[e + 2], v[e + 3]), M2, f2pack(A4.z, A4.w));
+          f2unpack(r0, v[e], v[e + 1]);
+          f2unpack(r1, v[e + 2], v[e + 3]);
         }
       };
       float gm[16];
 #pragma unroll
       for (int i = 0; i < 16; ++i) gm[i] = INFINITY;
+#pragma unroll 1
+      for (int cb = 0; cb < nchunk; cb += 2) {
+        float va[32], vb[32];
+        __syncwarp();
+        tmem_ld32x2(tD + lrow + cb * 32, tD + lrow + cb * 32 + 32, va, vb);
+        dt32(cb, va);
+        dt32(cb + 1, vb);
 #pragma unroll
-      for (int cb = 0; cb < 8; ++cb) {
-        if (cb < nchunk) {
-          float v[32];
-          load_dt(cb, v);
-#pragma unroll
-          for (int e = 0; e < 16; ++e) gm[e] = fmin3(gm[e], v[e], v[e + 16]);
-        }
+        for (int e = 0; e < 16; ++e) gm[e] = fmin3(fmin3(gm[e], va[e], va[e + 16]), vb[e], vb[e + 16]);
       }
-      float tq[CAP];
+      float tq[CAPT];
 #pragma unroll
-      for (int i = 0; i < CAP; ++i) tq[i] = INFINITY;
+      for (int i = 0; i < CAPT; ++i) tq[i] = INFINITY;
 #pragma unroll
       for (int gi = 0; gi < 16; ++gi) {  // sorted insertion, every slot from the old values
         const float x = gm[gi];
 #pragma unroll
-        for (int i = CAP - 1; i > 0; --i) tq[i] = fmaxf(tq[i - 1], fminf(tq[i], x));
+        for (int i = CAPT - 1; i > 0; --i) tq[i] = fmaxf(tq[i - 1], fminf(tq[i], x));
         tq[0] = fminf(tq[0], x);
       }
       const float T = sel_at(tq, Mc);
 
-      // [kList] entries of (dt, column) per row, slot-swizzled against bank conflicts
-      uint2* lst = reinterpret_cast<uint2*>(sA + row * 256);
-      const int sw = row & 31;
+      // [kList] entries of (dt, column) per row after a 32-float stash, slot-swizzled
+      uint8_t* rowbuf = sA + row * 256;
+      float* stash = reinterpret_cast<float*>(rowbuf);
+      uint2* lst = reinterpret_cast<uint2*>(rowbuf + 128);
+      const int sw = row & 7;
+      float tv[CAPT];
+      int tj[CAPT];
+#pragma unroll
+      for (int i = 0; i < CAPT; ++i) { tv[i] = INFINITY; tj[i] = 0x7FFFFFFF; }
       int cnt = 0;
 #pragma unroll 1
-      for (int cb = 0; cb < nchunk; ++cb) {
-        float v[32];
-        load_dt(cb, v);
+      for (int cb = 0; cb < nchunk; cb += 2) {
+        float va[32], vb[32];
+        __syncwarp();
+        tmem_ld32x2(tD + lrow + cb * 32, tD + lrow + cb * 32 + 32, va, vb);
+        dt32(cb, va);
+        dt32(cb + 1, vb);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          // branch-free: every column is written at the current slot, which
-          // advances only when the column is taken
-          lst[(cnt < kList ? cnt : kList - 1) ^ sw] = make_uint2(__float_as_uint(v[e]), (uint32_t)(cb * 32 + e));
-          cnt += v[e] <= T ? 1 : 0;
+        for (int hb = 0; hb < 2; ++hb) {
+          const float (&v)[32] = hb ? vb : va;
+          uint32_t mk = 0;
+#pragma unroll
+          for (int e = 0; e < 32; ++e) mk |= (v[e] <= T ? 1u : 0u) << e;
+          if (mk) {
+#pragma unroll
+            for (int k4 = 0; k4 < 8; ++k4)
+              reinterpret_cast<float4*>(stash)[k4 ^ sw] = make_float4(v[4 * k4], v[4 * k4 + 1], v[4 * k4 + 2], v[4 * k4 + 3]);
+            do {
+              const int e = __ffs(mk) - 1;
+              mk &= mk - 1;
+              const float x = stash[(((e >> 2) ^ sw) << 2) | (e & 3)];
+              const int j = (cb + hb) * 32 + e;
+              if (cnt < kList) lst[cnt] = make_uint2(__float_as_uint(x), (uint32_t)j);
+              ++cnt;
+              insert_top(tv, tj, Mc + 1, x, j);
+            } while (mk);
+          }
         }
       }
-      float tv[CAP];
-      int tj[CAP];
-#pragma unroll
-      for (int i = 0; i < CAP; ++i) { tv[i] = INFINITY; tj[i] = 0x7FFFFFFF; }
       const int mc = cnt < kList ? cnt : kList;
-      const int wmx = __reduce_max_sync(0xFFFFFFFFu, mc);
-      for (int i = 0; i < wmx; ++i)
-        if (i < mc) {
-          const uint2 en = lst[i ^ sw];
-          insert_top(tv, tj, Mc + 1, __uint_as_float(en.x), (int)en.y);
-        }
 
       const float kth = sel_at(tv, Mc - 1), nxt = sel_at(tv, Mc);
       const float kn = sqrtf(kn2);
@@ -362,7 +382,7 @@ __global__ void __launch_bounds__(FNT, 1)
       if (decided) {
 #pragma unroll
         for (int s = 0; s < kMaxFilterM; ++s)
-          if (s < Mc) myl[1 + s] = (uint8_t)tj[s];
+          if (s < Mc) myl[1 + s] = (uint8_t)tj[s < CAPT ? s : 0];
       }
       // The band (every j with dt_j <= kth + 2B, ascending j) of the rows
       // that are not decided: from the list when it covers the band
@@ -371,7 +391,7 @@ __global__ void __launch_bounds__(FNT, 1)
       if (need_band && lim <= T) {
         int c2 = 0;
         for (int i = 0; i < mc; ++i) {
-          const uint2 en = lst[i ^ sw];
+          const uint2 en = lst[i];
           const bool take = __uint_as_float(en.x) <= lim;
           const int sl = c2 < kBand ? c2 : kBand - 1;
           if (take) myl[1 + sl] = (uint8_t)en.y;
@@ -382,12 +402,17 @@ __global__ void __launch_bounds__(FNT, 1)
       const bool need_scan = need_band && !(lim <= T);
       if (__any_sync(0xFFFFFFFFu, need_scan)) {
         int c2 = 0;
-        for (int cb = 0; cb < nchunk; ++cb) {
-          float v[32];
-          load_dt(cb, v);
+#pragma unroll 1
+        for (int cb = 0; cb < nchunk; cb += 2) {
+          float va[32], vb[32];
+          __syncwarp();
+          tmem_ld32x2(tD + lrow + cb * 32, tD + lrow + cb * 32 + 32, va, vb);
+          dt32(cb, va);
+          dt32(cb + 1, vb);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const bool take = need_scan && v[e] <= lim;
+          for (int e = 0; e < 64; ++e) {
+            const float x = e < 32 ? va[e] : vb[e - 32];
+            const bool take = need_scan && x <= lim;
             const int sl = c2 < kBand ? c2 : kBand - 1;
             if (take) myl[1 + sl] = (uint8_t)(cb * 32 + e);
             c2 += take ? 1 : 0;
@@ -1114,12 +1139,14 @@ cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(append_filter, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
+    auto kern = a.M == 4 ? append_filter<5> : (a.M == 1 ? append_filter<2> : (a.M == 2 ? append_filter<3>
+                                                                                      : append_filter<kMaxFilterM + 1>));
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
     if (e != cudaSuccess) return e;
     const int tiles = (int)((a.N + 127) / 128);
     const int units = 2 * a.L.H * tiles;
     const int grid = units < nsm ? units : nsm;
-    append_filter<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
+    kern<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
