@@ -25,8 +25,9 @@
  *     asynchronous on it, except qwm_cache_status, which synchronises it.
  *   - Host-detectable errors (bad arguments, unsupported shapes, capacity)
  *     are returned before anything is launched.  Errors detected on the GPU
- *     (a bounded wait that ran out) are recorded in the cache's device status
- *     word, read with qwm_cache_status.
+ *     (a bounded wait that ran out; a value the binary16 operands cannot
+ *     hold) are recorded in the cache's device status word, read with
+ *     qwm_cache_status.
  *   - Supported: head_dim 128; group_size 32 or 64; 1 <= num_centroids <= 256;
  *     psac_rank 0, 8, 16 or 32; num_candidates >= 1 (values above
  *     num_centroids mean "all centroids"); scale_format 0 or 1.  Anything
@@ -72,7 +73,7 @@ typedef enum qwm_status {
   QWM_ERR_CAPACITY = 3,    /* chunk larger than a slot, or cache full without a window */
   QWM_ERR_CUDA = 4,        /* a CUDA runtime call failed */
   QWM_ERR_TIMEOUT = 5,     /* a bounded wait inside a kernel ran out (device status) */
-  QWM_ERR_NONFINITE = 6    /* reserved for non-finite inputs */
+  QWM_ERR_NONFINITE = 6    /* an input beyond the binary16 range or not a number (device status) */
 } qwm_status;
 
 /* Opaque host descriptor over a caller-owned device buffer. */
@@ -138,8 +139,26 @@ QWM_API qwm_status qwm_cache_chunk_info(const qwm_cache* cache, int32_t i, int32
 QWM_API qwm_status qwm_cache_layout(const qwm_cache* cache, qwm_layout* out);
 
 /* Synchronise `stream`, then read and clear the device status word: *status
- * receives QWM_OK or the first error a kernel recorded (QWM_ERR_TIMEOUT). */
+ * receives QWM_OK or the first error a kernel recorded (QWM_ERR_TIMEOUT,
+ * QWM_ERR_NONFINITE). */
 QWM_API qwm_status qwm_cache_status(qwm_cache* cache, int32_t* status, void* stream);
+
+/* Limit of every bounded wait inside the kernels that use this cache (an
+ * mbarrier wait between the roles of a kernel); default 2 s.  A wait that
+ * runs out makes its role leave its loop, the kernel finishes without further
+ * work on the GPU, and QWM_ERR_TIMEOUT is recorded in the status word (the
+ * outputs of that call are then incomplete).  1e3 <= ns <= 6e10, otherwise
+ * QWM_ERR_INVALID_ARG.  Host-side setting; applies to the calls made after it. */
+QWM_API qwm_status qwm_cache_set_wait_limit(qwm_cache* cache, uint64_t ns);
+
+/* Test hook of the timeout path (no counterpart in the paper): with role
+ * QWM_ROLE_V_REBUILD, the attention calls made afterwards leave the role that
+ * rebuilds V_hat idle, so the MMA warp's bounded wait for its first tile runs
+ * out (with a short qwm_cache_set_wait_limit, in milliseconds) and the call
+ * records QWM_ERR_TIMEOUT instead of computing.  0 restores normal work; any
+ * other role returns QWM_ERR_INVALID_ARG. */
+#define QWM_ROLE_V_REBUILD 1
+QWM_API qwm_status qwm_cache_set_idle_role(qwm_cache* cache, int32_t role);
 
 /* Scratch bytes qwm_fit_centroids needs for N tokens; 0 for an invalid
  * configuration.  With P = C rounded up to a multiple of 16 (at least 16),
@@ -190,7 +209,13 @@ QWM_API qwm_status qwm_fit_centroids_noalloc(const qwm_config* cfg, const void* 
  * (Eq. 15) or NULL to store no PSAC correction (cold start).  Keys: top-M
  * candidates by the Query-aware distance (Eq. 9), then the lowest QSAC score
  * (Eq. 12), ties to the lower index; Values: the same with w = 1 and no PSAC.
- * The chunk goes to the next slot (oldest slot when a sliding window is full). */
+ * The chunk goes to the next slot (oldest slot when a sliding window is full).
+ * The slot holds binary16 tables and scales and attention uses binary16
+ * operands: a Key, Value or centroid value of magnitude above 65504, or one
+ * that is not a number, or a group whose rebuilt values mu + s (q - z) could
+ * leave that range, records QWM_ERR_NONFINITE in the status word (the packed
+ * records are still written as defined above; rows with such values skip the
+ * tensor-core candidate filter and are decided on exact distances). */
 QWM_API qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* cache, const void* k, const void* v,
                                int64_t N, const void* k_centroids, const void* v_centroids,
                                const float* w, const void* U, void* stream);
@@ -203,9 +228,12 @@ QWM_API qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* cache, 
  * the past.  sm_scale > 0 (usually 1/sqrt(d)).
  * out: bf16 [Nq][H][d] = softmax(sm_scale * logits) V.
  * lse: fp32 [H][Nq] natural-log sum-exp of the scaled logits, or NULL.
- * The tensor-core operands are binary16 with fp32 accumulation, so q, k_cur,
- * v_cur and the rebuilt cache values must lie within the binary16 range
- * (|x| < 65504).
+ * The tensor-core operands are binary16 with fp32 accumulation, so q, k_cur
+ * and v_cur must lie within the binary16 range (|x| <= 65504): a finite value
+ * beyond it saturates to +-65504 (the output stays finite) and a NaN
+ * propagates; either records QWM_ERR_NONFINITE in the status word.  The
+ * rebuilt cache values are in range for every chunk whose append did not
+ * report QWM_ERR_NONFINITE.
  * At least one key (a cached chunk or N_cur > 0) is required. */
 QWM_API qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* cache, const void* q, int64_t Nq,
                       const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,

@@ -30,6 +30,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libqwm.so")
 
 QWM_OK = 0
+QWM_ROLE_V_REBUILD = 1
 STATUS_NAMES = {0: "QWM_OK", 1: "QWM_ERR_INVALID_ARG", 2: "QWM_ERR_UNSUPPORTED", 3: "QWM_ERR_CAPACITY",
                 4: "QWM_ERR_CUDA", 5: "QWM_ERR_TIMEOUT", 6: "QWM_ERR_NONFINITE"}
 
@@ -119,6 +120,10 @@ def lib():
             L.qwm_dequant_chunk.restype = ct.c_int
             L.qwm_top1_keys.argtypes = [_CFG, _P, ct.c_int64, _P, ct.c_int64, _P, _P]
             L.qwm_top1_keys.restype = ct.c_int
+            L.qwm_cache_set_wait_limit.argtypes = [_P, ct.c_uint64]
+            L.qwm_cache_set_wait_limit.restype = ct.c_int
+            L.qwm_cache_set_idle_role.argtypes = [_P, ct.c_int32]
+            L.qwm_cache_set_idle_role.restype = ct.c_int
             _lib = L
     return _lib
 
@@ -195,6 +200,14 @@ class Cache:
         lay = QwmLayout()
         _check("qwm_cache_layout", lib().qwm_cache_layout(self.handle, ct.byref(lay)))
         return lay
+
+    def set_wait_limit(self, ns: int):
+        """qwm_cache_set_wait_limit: limit of the kernels' bounded waits (ns)."""
+        _check("qwm_cache_set_wait_limit", lib().qwm_cache_set_wait_limit(self.handle, int(ns)))
+
+    def set_idle_role(self, role: int):
+        """qwm_cache_set_idle_role: test hook of the timeout path (0 = normal work)."""
+        _check("qwm_cache_set_idle_role", lib().qwm_cache_set_idle_role(self.handle, int(role)))
 
     def status(self) -> int:
         v = ct.c_int32()

@@ -374,9 +374,12 @@ __global__ void __launch_bounds__(FNT, 1)
       const float kn = sqrtf(kn2);
       const float Bb = ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
       const float lim = kth + 2.0f * Bb;
-      // a list overflow (more than kList columns at or below T) or a row out
-      // of the binary16 range is left to the exact rescoring of every centroid
-      const bool over = cnt > kList || !(kmx <= 65504.0f) || !(kn2 < INFINITY) || !(lim < INFINITY);
+      // a list overflow (more than kList columns at or below T), a row out of
+      // the binary16 range, or a table whose w o mu rows reach beyond it (the
+      // f16 operand would not hold them) is left to the exact rescoring of
+      // every centroid
+      const bool over = cnt > kList || !(kmx <= 65504.0f) || !(kn2 < INFINITY) || !(lim < INFINITY) ||
+                        !(Wn < 65504.0f);
       const bool decided = !over && nxt > lim;
       int n = over ? kRecAll : Mc;
       if (decided) {
@@ -543,6 +546,10 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
   }
   uint32_t ph = 0;
   int cur_pair = -1;
+  // A Key or Value or a table value beyond the binary16 range (or not a
+  // number) cannot be held by the cache's binary16 operands: reported in the
+  // cache's status word as QWM_ERR_NONFINITE once this CTA is done.
+  bool nbad = false;
 
   for (int u = u0; u < u1; ++u) {
     const int pair = u / tiles;
@@ -565,6 +572,7 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
       __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
       for (int i = tid; i < C * 64; i += QNT) {
         const uint32_t pr = src[i];
+        nbad |= bf16x2_out_of_f16(pr);
         dst[i] = __floats2half2_rn(__uint_as_float(pr << 16), __uint_as_float(pr & 0xFFFF0000u));
       }
       if (psac) {
@@ -874,6 +882,7 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
       // ---- 4. one channel pass: INT2 codes; Keys with PSAC also E (Eq. 4, 13),
       // c = U^T E, v = U^T (w o E) and err0 = sum_c w_c E_c^2, in channel order
       const uint64_t MAG2 = f2pack(kMagic, kMagic);
+      uint32_t kmag = 0u;  // the largest |k| bits of each half-word lane
       uint32_t mwn[8];
       ldg32(mr, mwn);
     #pragma unroll 1
@@ -891,6 +900,8 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
           const int ch = 2 * wd + hc;
           const uint4 kv = lds16(sK + sw_off(128, tid, ch));
           const uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
+          kmag = vmax_u16x2(vmax_u16x2(kmag, kv.x & 0x7FFF7FFFu), vmax_u16x2(kv.y & 0x7FFF7FFFu, kv.z & 0x7FFF7FFFu));
+          kmag = vmax_u16x2(kmag, kv.w & 0x7FFF7FFFu);
     #pragma unroll
           for (int p = 0; p < 4; ++p) {
             const uint64_t k2 = bf2_to_f2(kw[p]), m2 = bf2_to_f2(mw8[4 * hc + p]);
@@ -954,6 +965,13 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
         for (int i = 0; i < 8; ++i)
           if (i == wd) cw[i] = word;
       }
+      // |k0_c - k_c| <= s/2 (the INT2 round trip), so the rebuilt values stay
+      // inside the binary16 operands of attention when max|k| + s/2 does
+      {
+        const float km = fmaxf(__uint_as_float(kmag << 16), __uint_as_float(kmag & 0xFFFF0000u));
+        const float sm = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+        nbad |= bf16x2_out_of_f16(kmag) || !(km + 0.5f * sm < 65504.0f);
+      }
     }
     // every read of the tile is done: refill it with the next unit's tokens
     fence_proxy_async_smem();
@@ -1007,6 +1025,7 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
             for (int j = 0; j < R; ++j) amax = fmaxf(amax, fabsf(c[j]));
             const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
             const float sg = __half2float(sgh);
+            nbad |= !(127.0f * sg <= 65504.0f);  // C_hat = t sigma must stay a finite binary16
             const float sinv = sg != 0.0f ? __frcp_rn(sg) : 0.0f;
             float chat[R];
             uint32_t tq[R / 4];
@@ -1100,6 +1119,7 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
       }
     }
   }
+  if (nbad) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
 }
 
 // ============================================================================

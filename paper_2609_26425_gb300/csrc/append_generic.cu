@@ -12,10 +12,13 @@
 // contracted, and one __fmaf_rn per term of the sums of products), summed in
 // channel order, so the packed output is bit-exact against a sequential fp32
 // evaluation of the same formulas.
+#include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
 
 namespace qwm {
 namespace {
+
+using ptx::bf16x2_out_of_f16;
 
 constexpr int TT = 32;         // tokens per CTA
 constexpr int NT = 256;        // threads per CTA
@@ -82,11 +85,16 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
   // The chunk's own tables travel with the slot (one CTA per head and K/V),
   // stored as binary16 (exact for bf16 values in the binary16 range), the
   // operand type of the attention kernel's tensor-core path.
+  // A Key or Value or a table value beyond the binary16 range (or not a
+  // number) cannot be held by the cache's binary16 operands: reported in the
+  // cache's status word as QWM_ERR_NONFINITE.
+  bool nbad = false;
   if (blockIdx.x == 0) {
     const uint32_t* src = reinterpret_cast<const uint32_t*>(tab);
     __half2* dst = reinterpret_cast<__half2*>(head + (is_key ? L.ktab : L.vtab));
     for (int i = tid; i < C * 64; i += NT) {
       const uint32_t pr = src[i];
+      nbad |= bf16x2_out_of_f16(pr);
       dst[i] = __floats2half2_rn(bf_lo(pr), bf_hi(pr));
     }
     if (psac) {
@@ -108,12 +116,16 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
     const int ti = i >> 6, wd = i & 63;
     const int64_t t = t0 + ti;
     uint32_t pr = 0;
-    if (t < a.N) pr = reinterpret_cast<const uint32_t*>(x + ((size_t)t * H + h) * 128)[wd];
+    if (t < a.N) {
+      pr = reinterpret_cast<const uint32_t*>(x + ((size_t)t * H + h) * 128)[wd];
+      nbad |= bf16x2_out_of_f16(pr);
+    }
     s.x[ti * 128 + 2 * wd] = bf_lo(pr);
     s.x[ti * 128 + 2 * wd + 1] = bf_hi(pr);
   }
   if (psac)
     for (int i = tid; i < 128 * r; i += NT) s.U[i] = a.U[(size_t)h * 128 * r + i];  // [d][r]
+  if (nbad) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
   __syncthreads();
   if (tid < ng) {
     float Wg = 0.0f;
@@ -265,6 +277,9 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
         k0[e] = __fadd_rn(mu4[e], __fmul_rn((float)(q - z), sc));
       }
     }
+    // the rebuilt values must stay inside the binary16 operands of attention
+    if (!(fmaxf(fmaxf(fabsf(k0[0]), fabsf(k0[1])), fmaxf(fabsf(k0[2]), fabsf(k0[3]))) < 65504.0f))
+      atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
     uint32_t zbyte = 0;
     for (int g = 0; g < ng; ++g) zbyte |= (uint32_t)__shfl_sync(0xFFFFFFFFu, z, g * glanes) << (2 * g);
 
@@ -323,6 +338,8 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
         for (int off = 16; off; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, off));
         const __half sgh = __float2half_ru(__fdiv_rn(amax, 127.0f));
         const float sg = __half2float(sgh);
+        if (lane == 0 && !(127.0f * sg <= 65504.0f))  // C_hat = t sigma must stay a finite binary16
+          atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
         int tq = 0;
         float ch = 0.0f;
         if (sg != 0.0f && lane < r) {

@@ -66,7 +66,7 @@ constexpr int UBLK = 4096;                 // 32 rows x 128 bytes
 constexpr int OFF_BAR = OFF_U + 4 * UBLK;
 enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_PFULL = 10, B_QU = 12, B_OFINAL = 14,
        B_QUMMA = 15, NBAR = 17 };
-static_assert(NBAR * 8 + 12 <= 256, "barrier area");
+static_assert(NBAR * 8 + 16 <= 256, "barrier area");
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;  // + alignment slack
 
 // 8 f16 (16 bytes) of row `row`, chunk `ch` (columns 8ch..8ch+7) into a run of
@@ -101,11 +101,6 @@ __device__ __forceinline__ uint64_t splat2(float a) {
   asm("mov.b64 %0, {%1, %1};" : "=l"(x) : "f"(a));
   return x;
 }
-__device__ __forceinline__ float fmax3(float a, float b, float c) {
-  float m;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(m) : "f"(a), "f"(b), "f"(c));
-  return m;
-}
 
 // 32-byte read-only global load (address 32-byte aligned).
 __device__ __forceinline__ void ldg32B(const void* p, uint32_t (&r)[8]) {
@@ -121,10 +116,13 @@ __device__ __forceinline__ void zero_row(uint8_t* dst, int row, int ch0, int nch
   for (int ch = ch0; ch < ch0 + nch; ++ch) st_chunk(dst, row, ch, make_uint4(0, 0, 0, 0));
 }
 
-__device__ __forceinline__ void copy_row(uint8_t* dst, int row, const __nv_bfloat16* src) {
+// A row of 128 bf16 into the f16 operand; values beyond the binary16 range
+// saturate and set `bad`.
+__device__ __forceinline__ void copy_row(uint8_t* dst, int row, const __nv_bfloat16* src, bool& bad) {
 #pragma unroll
-  for (int ch = 0; ch < 16; ++ch) st_chunk(dst, row, ch, bf16x8_to_f16x8(ldg16(src + ch * 8)));
+  for (int ch = 0; ch < 16; ++ch) st_chunk(dst, row, ch, bf16x8_to_f16x8_sat(ldg16(src + ch * 8), bad));
 }
+
 
 struct Unit {
   int ntok;
@@ -210,6 +208,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + OFF_BAR + NBAR * 8);
   int* s_err = reinterpret_cast<int*>(sm + OFF_BAR + NBAR * 8 + 8);
+  volatile int* s_bad = reinterpret_cast<volatile int*>(sm + OFF_BAR + NBAR * 8 + 12);  // an input beyond binary16
   auto bar = [&](int i) { return smem_u32(bars + i); };
   // One arrival per warp on the leader's copy of barrier i, after every lane's
   // writes (the caller fences them for their consumer first).
@@ -252,6 +251,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     mbar_init(bar(B_QUMMA), 1);         // Q_i U_r MMA commit, both CTAs
     mbar_init(bar(B_QUMMA + 1), 1);
     *s_err = 0;
+    *s_bad = 0;
     fence_mbar_init();
   }
   if (warp == W_MMA) {
@@ -273,8 +273,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     const uint32_t tS = tbase + 128 * i + lrow, tO = tbase + 256 + 128 * i + lrow;
     const __nv_bfloat16* qrow = a.q + ((size_t)(qvalid ? qi : 0) * H + h) * 128;
     uint8_t* sQi = sm + OFF_Q + i * 2 * BLK;
-    if (qvalid) copy_row(sQi, row, qrow);
+    bool qbad = false;
+    if (qvalid) copy_row(sQi, row, qrow, qbad);
     else zero_row(sQi, row, 0, 16);
+    if (qbad) *s_bad = 1;
     fence_proxy_async_smem();
     arrive_leader(B_QU + i);  // Q_i is in place
     // Q_i U_r of each chunk that carries PSAC columns: the MMA thread computes
@@ -283,7 +285,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     if (i < nqt) {
     uint32_t qum = 0;  // completed Q_i U_r MMAs
     auto take_qu = [&]() -> bool {
-      bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1));
+      bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_QUMMA + i), qum & 1, a.wait_ns));
       if (okw) {
         ++qum;
         tc_fence_after();
@@ -306,7 +308,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int ntiles = (U.ntok + 127) / 128;
       for (int tl = 0; tl < ntiles; ++tl, ++jt) {
         const int nvalid = min(128, U.ntok - tl * 128);
-        const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1));
+        const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL + i), jt & 1, a.wait_ns));
         if (okw) {
           tc_fence_after();
           // ---- row maximum: four reducing TMEM loads and one wait
@@ -396,7 +398,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       }
       if (ok && u + 1 < n_units && unit_at(a, S, u + 1, h).psac) ok = take_qu();
     }
-    if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFINAL), 0));
+    if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFINAL), 0, a.wait_ns));
     if (ok) {
       tc_fence_after();
       const float inv_l = 1.0f / l_run;
@@ -417,6 +419,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       if (a.lse && qvalid) a.lse[(size_t)h * a.Nq + qi] = m_run * a.sm_scale + logf(l_run);
     } else {
       *s_err = 1;
+    }
+    // Off the critical path: this CTA's share of the active chunk's rows of
+    // head h (the rebuild converts them with saturation) is checked for values
+    // beyond the binary16 range, which only the status word reports.
+    if (a.Ncur > 0) {
+      const int64_t per = (a.Ncur + gridDim.x - 1) / gridDim.x;
+      const int64_t r0 = (int64_t)blockIdx.x * per, r1 = min(a.Ncur, r0 + per);
+      uint32_t mag = 0u;
+      for (int64_t e = r0 * 16 + (tid & 255); e < r1 * 16; e += 256) {
+        const int64_t tok = e >> 4;
+        const int ch = (int)(e & 15);
+        const uint4 kv = ldg16(a.kcur + ((size_t)tok * H + h) * 128 + ch * 8);
+        const uint4 vv = ldg16(a.vcur + ((size_t)tok * H + h) * 128 + ch * 8);
+        const uint32_t w8[8] = {kv.x, kv.y, kv.z, kv.w, vv.x, vv.y, vv.z, vv.w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mag = vmax_u16x2(mag, w8[i] & 0x7FFF7FFFu);
+      }
+      if (bf16x2_out_of_f16(mag)) *s_bad = 1;
     }
     }
   } else if (warp < W_DQV) {
@@ -460,7 +480,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
-      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_KEMPTY + st), ph ^ 1));
+      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_KEMPTY + st), ph ^ 1, a.wait_ns));
       if (okw) {
         uint8_t* dst = sm + OFF_K + 2 * st * HBLK;
         const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
@@ -473,7 +493,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   #pragma unroll 1
           for (int idx = kt; idx < 32 * 16; idx += 128) {
             const int j = idx >> 4, ch = idx & 15;
-            const uint4 v = j < r ? bf16x8_to_f16x8(ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2)) : make_uint4(0u, 0u, 0u, 0u);
+            bool ubad = false;
+            const uint4 v = j < r ? bf16x8_to_f16x8_sat(ldg16(ut + ((int64_t)j * 128 + ch * 8) * 2), ubad) : make_uint4(0u, 0u, 0u, 0u);
+            if (ubad) *s_bad = 1;
             st_chunk(sU, j, ch, v, 32);
           }
         }
@@ -588,7 +610,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     const int wrow = (warp & 3) * 32 + rr;  // row of pass p: wrow + 8p
     const int c16 = 4 * (int)rank + q;      // this lane's 16-channel block of the row
     TileCursor cur;
-    cur.init(a, S, h, n_units);
+    // an idle V role (the test hook of qwm_cache_set_idle_role) publishes no
+    // tile: the MMA warp's bounded wait for the first one runs out
+    cur.init(a, S, h, a.idle_role == QWM_ROLE_V_REBUILD ? 0 : n_units);
     auto load_ids = [&](const TileCursor& c) -> uint64_t {  // 4 ids | 4 zero bytes << 32
       uint64_t v = 0;
       if (c.valid() && c.U.hb) {
@@ -613,7 +637,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       const int st = jt & 1;
       const uint32_t ph = (jt >> 1) & 1;
       const int nv = cur.nvalid();
-      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_VEMPTY + st), ph ^ 1));
+      const bool okw = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_VEMPTY + st), ph ^ 1, a.wait_ns));
       if (okw) {
         uint8_t* dst = sm + OFF_V + st * BLK;
         const uint8_t* tb = cur.U.hb ? cur.U.hb + L.tiles_off + (int64_t)cur.tl * L.tile_bytes : nullptr;
@@ -701,9 +725,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       auto issue_S = [&](int i) -> bool {
         const int st = sjt & 1;
         const uint32_t ph = (sjt >> 1) & 1;
-        if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph)) return false;
+        if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph, a.wait_ns)) return false;
         if (sc.tl == 0 && sc.u == 0) {  // Q_i in place
-          if (!mbar_wait_cluster(bar(B_QU + i), qph[i])) return false;
+          if (!mbar_wait_cluster(bar(B_QU + i), qph[i], a.wait_ns)) return false;
           qph[i] ^= 1;
         }
         if (sc.tl == 0 && sc.U.psac) {
@@ -719,7 +743,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
               umma2_ss(tbase + 128 * i + 64, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
                        desc_sw128(aUc + kb * UBLK + ks * 32), idQU, (kb | ks) != 0);
           umma2_commit_both(bar(B_QUMMA + i));
-          if (!mbar_wait_cluster(bar(B_QU + i), qph[i])) return false;  // moved into the shared A operand
+          if (!mbar_wait_cluster(bar(B_QU + i), qph[i], a.wait_ns)) return false;  // moved into the shared A operand
           qph[i] ^= 1;
         }
         tc_fence_after();
@@ -745,10 +769,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       for (int jt = 0; jt < total && ok; ++jt) {
         const int st = jt & 1;
         const uint32_t ph = (jt >> 1) & 1;
-        if (!(ok = mbar_wait_cluster(bar(B_VFULL + st), ph))) break;
+        if (!(ok = mbar_wait_cluster(bar(B_VFULL + st), ph, a.wait_ns))) break;
 #pragma unroll
         for (int i = 0; i < nqt; ++i) {
-          if (!(ok = mbar_wait_cluster(bar(B_PFULL + i), jt & 1))) break;
+          if (!(ok = mbar_wait_cluster(bar(B_PFULL + i), jt & 1, a.wait_ns))) break;
           tc_fence_after();
           const uint32_t tP = tbase + 128 * i, tO = tbase + 256 + 128 * i;
 #pragma unroll
@@ -759,7 +783,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
       }
       umma2_commit_both(bar(B_OFINAL));
-      if (!ok) *s_err = 1;
+      if (!ok) {
+        // a wait ran out: let the MMAs already issued finish before the
+        // pair's TMEM is released
+        mbar_wait(bar(B_OFINAL), 0, a.wait_ns);
+        *s_err = 1;
+      }
     }
     __syncwarp();
   }
@@ -767,6 +796,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   tc_fence_before();
   __syncthreads();
   if (tid == 0 && *s_err) atomicCAS(a.status, 0, (int)QWM_ERR_TIMEOUT);
+  if (tid == 0 && *s_bad) atomicCAS(a.status, 0, (int)QWM_ERR_NONFINITE);
   cluster_sync();  // neither CTA frees the pair's TMEM while the other still reads it
   if (warp == W_MMA) {
     tc_fence_after();

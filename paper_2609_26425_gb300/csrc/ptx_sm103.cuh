@@ -409,12 +409,49 @@ __device__ __forceinline__ uint32_t pack_f16(float a, float b) {
   __half2 h = __floats2half2_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
 }
-// 8 bf16 -> 8 f16 (exact for |x| in the binary16 normal range).
+// 8 bf16 -> 8 f16 (exact for |x| in the binary16 normal range; a finite value
+// beyond it saturates to +-65504, a NaN stays NaN).  cvt.f16x2 puts its first
+// source in the upper half.
 __device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 v) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
   uint32_t o[4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) o[i] = pack_f16(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+  for (int i = 0; i < 4; ++i)
+    asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;"
+        : "=r"(o[i]) : "f"(__uint_as_float(w[i] & 0xFFFF0000u)), "f"(__uint_as_float(w[i] << 16)));
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// Lane-wise maximum of two pairs of 16-bit unsigned integers.
+__device__ __forceinline__ uint32_t vmax_u16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.u16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+// 16-bit halves of a bf16 pair whose magnitude is at least 2^16 (the first
+// bf16 value above the largest binary16, 65504) or which are inf/NaN: true
+// when either half is outside the binary16 range.
+__device__ __forceinline__ bool bf16x2_out_of_f16(uint32_t w) {
+  const uint32_t m = w & 0x7FFF7FFFu;
+  return (m & 0xFFFFu) >= 0x4780u || (m >> 16) >= 0x4780u;
+}
+// 8 bf16 -> 8 f16 like bf16x8_to_f16x8, but a value outside the binary16
+// range becomes +-65504 (a NaN becomes -65504) and sets `bad`: the result then
+// differs from the input, and the caller reports it.  One magnitude test per
+// 8 values; the clamping conversion runs only when it fails.
+__device__ __forceinline__ uint4 bf16x8_to_f16x8_sat(uint4 v, bool& bad) {
+  const uint32_t m = vmax_u16x2(vmax_u16x2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu),
+                                vmax_u16x2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu));
+  if (!bf16x2_out_of_f16(m)) return bf16x8_to_f16x8(v);
+  bad = true;
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float lo = fminf(fmaxf(__uint_as_float(w[i] << 16), -65504.0f), 65504.0f);
+    const float hi = fminf(fmaxf(__uint_as_float(w[i] & 0xFFFF0000u), -65504.0f), 65504.0f);
+    o[i] = pack_f16(lo, hi);
+  }
   return make_uint4(o[0], o[1], o[2], o[3]);
 }
 

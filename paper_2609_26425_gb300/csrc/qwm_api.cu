@@ -60,6 +60,8 @@ struct qwm_cache {
   int64_t appended;                       // chunks appended so far
   int32_t n_tokens[qwm::kMaxSlots];       // tokens held by each slot
   int32_t psac[qwm::kMaxSlots];           // slot stored with a PSAC correction
+  uint64_t wait_ns;                       // limit of the kernels' bounded waits
+  int32_t idle_role;                      // qwm_cache_set_idle_role (0: none)
 };
 
 namespace {
@@ -127,6 +129,8 @@ qwm_status qwm_cache_init(qwm_cache** out, const qwm_config* cfg, void* dev_buf,
   c->bytes = bytes;
   c->sliding_window = sliding_window;
   c->appended = 0;
+  c->wait_ns = 2000000000ull;
+  c->idle_role = 0;
   if (cudaMemsetAsync(dev_buf, 0, qwm::kHeaderBytes, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
     delete c;
     return QWM_ERR_CUDA;
@@ -301,7 +305,21 @@ qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, 
   a.sm_scale = sm_scale;
   a.out = static_cast<__nv_bfloat16*>(out);
   a.lse = lse;
+  a.wait_ns = c->wait_ns;
+  a.idle_role = c->idle_role;
   return qwm::launch_attend(a, slots, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
+}
+
+qwm_status qwm_cache_set_wait_limit(qwm_cache* c, uint64_t ns) {
+  if (!c || ns < 1000ull || ns > 60000000000ull) return QWM_ERR_INVALID_ARG;
+  c->wait_ns = ns;
+  return QWM_OK;
+}
+
+qwm_status qwm_cache_set_idle_role(qwm_cache* c, int32_t role) {
+  if (!c || (role != 0 && role != QWM_ROLE_V_REBUILD)) return QWM_ERR_INVALID_ARG;
+  c->idle_role = role;
+  return QWM_OK;
 }
 
 }  // extern "C"

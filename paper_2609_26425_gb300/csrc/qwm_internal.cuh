@@ -127,6 +127,8 @@ struct AttendArgs {
   float sm_scale;
   __nv_bfloat16* out;          // [Nq][H][d]
   float* lse;                  // [H][Nq] or null
+  uint64_t wait_ns;            // limit of every bounded wait
+  int32_t idle_role;           // QWM_ROLE_*: a role that publishes nothing (test hook), 0 = none
 };
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t s);
 

@@ -75,3 +75,10 @@ def oracle_kv(ko: dict, vo: dict, kc_bits, vc_bits, *, G, r, U_bits=None):
     K = orc.dequant(ko, kc_bits, G=G, r=r, U_bits=U_bits if r > 0 else None)
     V = orc.dequant(vo, vc_bits, G=G, r=0)
     return K, V
+
+
+def strided_centroids(x_bits, C):
+    """Generator-side centroid table: tokens floor(j*N/C) of the chunk (no arithmetic)."""
+    N = x_bits.shape[0]
+    idx = (np.arange(C) * N) // C
+    return np.ascontiguousarray(x_bits[idx].transpose(1, 0, 2))

@@ -138,3 +138,11 @@ def test_fit_entry_points_accept_the_same_configurations(qlib):
         assert L.qwm_fit_centroids(ct.byref(bad), fake, 10, fake, fake, 1 << 30, None) == 2
         assert fn(ct.byref(bad), fake, 10, fake, None) == 2
     assert fn(ct.byref(qlib.config(4, 64)), fake, 0, fake, None) == 1
+
+
+def test_wait_limit_and_idle_role_argument_checks(qlib):
+    """The timeout-path settings reject a missing cache and values out of range
+    without touching a device."""
+    L = qlib.lib()
+    assert L.qwm_cache_set_wait_limit(None, 1_000_000) == 1
+    assert L.qwm_cache_set_idle_role(None, 0) == 1

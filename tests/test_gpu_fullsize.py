@@ -204,3 +204,44 @@ def test_microbench_sweep_extremes(H, chunks, C, G, r, Nq, Ncur):
                               1 / math.sqrt(128), rows=rows)
     compare_attention(out.float().cpu().numpy()[rows][:, heads], ref)
     assert np.abs(lse.cpu().numpy()[heads][:, rows] - ref_lse).max() < 2e-2
+
+
+def test_wan14b_append_with_fitted_tables_sampled_heads():
+    """The bench's append configuration with k-means tables: the Wan-14B chunk
+    (40 heads, 4680 tokens, C = 256, 10 Lloyd iterations).  Three heads take
+    the oracle's own fitted tables (many near ties between centroids, unlike
+    strided tokens); the other heads take the GPU's fit, which the k-means
+    parity tests prove equal to the oracle's.  Sampled tokens of the three
+    heads are compared with the oracle bit for bit under the margin rule."""
+    wl = synth.WORKLOADS["wan14b_layer"]
+    H, N, C, G, r, M = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.psac_rank, wl.candidates
+    heads = [0, 17, 39]
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, kmeans_iters=wl.kmeans_iters)
+    src = synth.ChunkSource(wl)
+    _, k, v = src.chunk(wl.past_chunks)
+    a = src.query_log_scale(wl.past_chunks)
+    w = synth.population_w(a).numpy()
+    Ub = synth.bits(synth.population_U(a, r))
+    kb, vb = synth.bits(k), synth.bits(v)
+    kd, vd = dev(k), dev(v)
+    kc_g = synth.bits(qwm.qwm_fit_centroids(cfg, kd).cpu())
+    vc_g = synth.bits(qwm.qwm_fit_centroids(cfg, vd).cpu())
+    kc_o = orc.fit_centroids(np.ascontiguousarray(kb[:, heads]), C, wl.kmeans_iters)["centroids"]
+    vc_o = orc.fit_centroids(np.ascontiguousarray(vb[:, heads]), C, wl.kmeans_iters)["centroids"]
+    kc, vc = kc_g.copy(), vc_g.copy()
+    kc[heads], vc[heads] = kc_o, vc_o
+    cache = qwm.Cache(cfg, N, 1)
+    qwm.qwm_quantize_append(cfg, cache, kd, vd, dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
+                            w=torch.from_numpy(w).cuda(), U=dev(synth.from_bits(Ub)))
+    torch.cuda.synchronize()
+    assert cache.status() == 0
+    dec = cache.decode_chunk(0)
+    idx = sample_rows(N, 160, 77)
+    hs = np.array(heads)
+    g = {key: dec[key][idx][:, hs] for key in ("ids", "codes", "scales", "zeros", "coef", "sigma",
+                                               "v_ids", "v_codes", "v_scales", "v_zeros")}
+    kbs = np.ascontiguousarray(kb[idx][:, hs])
+    vbs = np.ascontiguousarray(vb[idx][:, hs])
+    ko, vo = oracle_append(kbs, vbs, kc_o, vc_o, G=G, r=r, M=M, w=w[hs], U_bits=Ub[hs])
+    compare_packed(g, ko, kbs, kc_o, G=G, r=r, M=M, is_key=True, w=w[hs], U_bits=Ub[hs])
+    compare_packed(g, vo, vbs, vc_o, G=G, r=r, M=M, is_key=False, prefix="v_")

@@ -17,7 +17,7 @@ from oracle import oracle as orc
 from paper_2609_26425_gb300 import synth
 import paper_2609_26425_gb300 as qwm
 
-from parity import compare_attention, compare_packed, oracle_append, oracle_kv
+from parity import compare_attention, compare_packed, oracle_append, oracle_kv, strided_centroids
 
 pytestmark = pytest.mark.gpu
 
@@ -37,13 +37,6 @@ def f16_bits(bf16_bits):
     """bf16 bit patterns -> binary16 bit patterns of the same values (torch conversion)."""
     t = synth.from_bits(bf16_bits).to(torch.float16)
     return t.view(torch.int16).numpy().view(np.uint16)
-
-
-def strided_centroids(x_bits, C):
-    """Generator-side centroid table: tokens floor(j*N/C) of the chunk (no arithmetic)."""
-    N = x_bits.shape[0]
-    idx = (np.arange(C) * N) // C
-    return np.ascontiguousarray(x_bits[idx].transpose(1, 0, 2))
 
 
 def make_chunk(seed, N, H, *, outliers=True):
