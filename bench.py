@@ -464,6 +464,225 @@ def query_stats_timing(qwm, cfg, qd, dev, iters, stream):
     return {"update_ms": upd, "basis_ms": bas, "update_bytes": nbytes, "sweeps": st.sweeps()}
 
 
+# ---------------------------------------------------------------------------- layer stacks
+def stack_flops(wl, r, cached_tokens):
+    """Attend FLOPs of one chunk step over every layer of a stack."""
+    H, N, d = wl.heads, wl.chunk_tokens, wl.head_dim
+    return wl.layers * 2.0 * H * N * (cached_tokens * (2 * d + r) + N * 2 * d)
+
+
+def run_stack(args, wl, psac_rank=None, distinct_layers=4):
+    """Per-chunk time of a stack of layers: at every chunk step, each layer's
+    new chunk attends its cached chunks and itself (bf16), then is appended;
+    the step's times are summed over the layers (CUDA events around each
+    call), with the packed bytes the caches hold against bf16 K/V of the same
+    tokens.  Layer l draws the seeded inputs of layer l mod distinct_layers
+    (the timing does not depend on the draw; drawing every layer's inputs on
+    the host would take minutes).  Centroid tables: the GPU k-means of each
+    chunk (10 Lloyd iterations)."""
+    import torch
+    import paper_2609_26425_gb300 as qwm
+    from paper_2609_26425_gb300 import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    qwm.lib()
+    r = wl.psac_rank if psac_rank is None else psac_rank
+    H, N, C, G, M, d = wl.heads, wl.chunk_tokens, wl.centroids, wl.group_size, wl.candidates, wl.head_dim
+    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=M, kmeans_iters=wl.kmeans_iters,
+                     scale_format=args.scale_format)
+    # without a window the last step attends past_chunks chunks and then
+    # appends one more; a window wraps around for two more steps at the end
+    slots = wl.window if wl.window else wl.past_chunks + 1
+    n_chunks = wl.past_chunks + (3 if wl.window else 1)
+    Dl = min(distinct_layers, wl.layers)
+    ws = torch.empty(qwm.qwm_fit_workspace_bytes(cfg, N), dtype=torch.uint8, device=dev)
+    data = []
+    for layer in range(Dl):
+        src = synth.ChunkSource(wl, layer=layer)
+        row = []
+        for t in range(n_chunks):
+            q, k, v = src.chunk(t)
+            a = src.query_log_scale(t)
+            qd, kd, vd = q.to(dev), k.to(dev), v.to(dev)
+            kc = qwm.qwm_fit_centroids(cfg, kd, workspace=ws)
+            vc = qwm.qwm_fit_centroids(cfg, vd, workspace=ws)
+            w = synth.population_w(a).to(dev) if t > 0 else None
+            U = synth.population_U(a, r).to(dev) if (t > 0 and r > 0) else None
+            row.append((qd, kd, vd, kc, vc, w, U))
+        data.append(row)
+    caches = [qwm.Cache(cfg, N, slots, sliding_window=bool(wl.window), device=dev) for _ in range(wl.layers)]
+    stream = torch.cuda.current_stream()
+    out = torch.empty(N, H, d, dtype=torch.bfloat16, device=dev)
+    for layer in range(wl.layers):   # chunk 0, cold start (w = 1, no PSAC): append only
+        _, kd, vd, kc, vc, w, U = data[layer % Dl][0]
+        qwm.qwm_quantize_append(cfg, caches[layer], kd, vd, kc, vc, w=w, U=U)
+    for _ in range(3):                # warm-up of the attention path
+        qwm.qwm_attend(cfg, caches[0], data[0][1][0], data[0][1][1], data[0][1][2], out=out)
+    torch.cuda.synchronize()
+    lay = caches[0].layout()
+    clocks = ClockSampler(0)
+    clocks.start()
+    rows = []
+    for t in range(1, n_chunks):
+        cached = caches[0].num_chunks
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(wl.layers)]
+        for layer in range(wl.layers):
+            qd, kd, vd, kc, vc, w, U = data[layer % Dl][t]
+            evs[layer][0].record(stream)
+            qwm.qwm_attend(cfg, caches[layer], qd, kd, vd, out=out)
+            evs[layer][1].record(stream)
+            qwm.qwm_quantize_append(cfg, caches[layer], kd, vd, kc, vc, w=w, U=U)
+            evs[layer][2].record(stream)
+        torch.cuda.synchronize()
+        att = sum(e[0].elapsed_time(e[1]) for e in evs)
+        app = sum(e[1].elapsed_time(e[2]) for e in evs)
+        held = caches[0].num_chunks
+        flops = stack_flops(wl, r, cached * N)
+        nums = workload_numbers(wl, args.scale_format)
+        rows.append({"step": t, "cached_tokens": cached * N, "attend_ms": round(att, 3), "append_ms": round(app, 3),
+                     "attend_tflops": round(flops / (att * 1e-3) / 1e12, 1),
+                     "append_gbs": round(wl.layers * nums["append_bytes"] / (app * 1e-3) / 1e9, 1),
+                     "cache_gib": round(wl.layers * (lay.header_bytes + held * lay.slot_bytes) / 2**30, 3),
+                     "bf16_gib": round(wl.layers * held * N * H * d * 2 * 2 / 2**30, 3)})
+    clk = clocks.stop()
+    for c in caches:
+        if c.status():
+            raise RuntimeError("device status after the stack run")
+    return rows, clk, r
+
+
+def stack_line(args, wl, psac_rank=None):
+    rows, clk, r = run_stack(args, wl, psac_rank)
+    pk = peaks()
+    # a window: the steps with the window full; no window: the last step
+    full = [x for x in rows if x["cached_tokens"] == wl.window * wl.chunk_tokens] if wl.window else rows[-1:]
+    last = full[-1] if full else rows[-1]
+    att_ms = sum(x["attend_ms"] for x in full) / len(full)
+    app_ms = sum(x["append_ms"] for x in full) / len(full)
+    flops = stack_flops(wl, r, last["cached_tokens"])
+    tflops = flops / (att_ms * 1e-3) / 1e12
+    nums = workload_numbers(wl, args.scale_format)
+    res = {
+        "metric": METRIC, "value": round(tflops, 3), "unit": UNIT, "n_gpus": 1, "steps": len(rows), "warmup": 3,
+        "ms_per_step": round(att_ms + app_ms, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "config": {"workload": wl.name, "layers": wl.layers, "heads": wl.heads, "chunk_tokens": wl.chunk_tokens,
+                   "cache_chunks": wl.window or wl.past_chunks, "sliding_window": bool(wl.window),
+                   "centroids": wl.centroids, "group_size": wl.group_size, "psac_rank": r,
+                   "candidates": wl.candidates, "inputs": "4 seeded layers cycled over the stack",
+                   "value": ("mean over the steps with a full window" if wl.window else "the last step (the full cache)") +
+                            ": attend FLOPs of all layers / summed attend time"},
+        "attend": {"ms": round(att_ms, 3), "tflops": round(tflops, 2),
+                   "frac_of_measured_bf16": round(tflops / pk["bf16_tflops"], 4)},
+        "append": {"ms": round(app_ms, 3),
+                   "gbs": round(wl.layers * nums["append_bytes"] / (app_ms * 1e-3) / 1e9, 1),
+                   "frac_of_measured_hbm": round(wl.layers * nums["append_bytes"] / (app_ms * 1e-3) / 1e9 /
+                                                 pk["hbm_gbs"], 4)},
+        "roofline": {"bound": "tensor", "kernel": "attend_kernel", "achieved": round(tflops, 2),
+                     "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": round(tflops / pk["bf16_tflops"], 4),
+                     "traffic": None, "peak_src": pk["src"] + " burst bf16"},
+        "gpu_launches": (1 + 2) * wl.layers * len(rows),
+        "clocks": clk, "per_step": rows,
+    }
+    if not args.no_cpu_baseline:
+        cb = cpu_baseline(wl, args.cpu_threads, f=0.25, f_single=0.02)
+        cb["note"] = "one layer's step sampled (every layer does the same work per FLOP)"
+        res["cpu_baseline"] = cb
+    return res
+
+
+# ---------------------------------------------------------------------------- microbench sweep
+def run_sweep(args, Ns=(1024, 4096, 16384, 65536), Ls=(4096, 16384, 65536, 131072), Cs=(16, 64, 256),
+              rs=(0, 8, 16, 32), Gs=(32, 64), H=40, reps=3):
+    """The one-layer microbench sweep (40 heads): attend over every N x L x r
+    (C = 256, G = 32; N_q = N_cur = N; caches built from 4096-token chunks),
+    and quantize-append over every N x C x r x G (k-means tables of the chunk,
+    10 Lloyd iterations); each point timed with CUDA events after an L2
+    flush, as throughput and fraction of the measured roofline."""
+    import torch
+    import paper_2609_26425_gb300 as qwm
+    from paper_2609_26425_gb300 import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    qwm.lib()
+    pk = peaks()
+    d = 128
+    wl = synth.Workload("sweep", heads=H, chunk_tokens=max(Ns), past_chunks=0, centroids=256, group_size=32,
+                        psac_rank=16, seed=4)
+    src = synth.ChunkSource(wl)
+    q, k, v = src.chunk(0)
+    a = src.query_log_scale(0)
+    qd, kd, vd = q.to(dev), k.to(dev), v.to(dev)
+    w = synth.population_w(a).to(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        ms = []
+        for _ in range(reps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        return sorted(ms)[len(ms) // 2]
+
+    attend_pts = []
+    Lc = 4096
+    for r in rs:
+        cfg = qwm.config(H, 256, group_size=32, psac_rank=r, candidates=4)
+        U = synth.population_U(a, r).to(dev) if r > 0 else None
+        cache = qwm.Cache(cfg, Lc, max(Ls) // Lc, device=dev)
+        kc = kd[: 256 * (Lc // 256): Lc // 256].transpose(0, 1).contiguous()   # strided tokens as tables
+        vc = vd[: 256 * (Lc // 256): Lc // 256].transpose(0, 1).contiguous()
+        for i in range(max(Ls) // Lc):
+            o = (i % (max(Ns) // Lc)) * Lc
+            qwm.qwm_quantize_append(cfg, cache, kd[o:o + Lc], vd[o:o + Lc], kc, vc, w=w, U=U)
+            L = (i + 1) * Lc
+            if L in Ls:
+                for N in Ns:
+                    out = torch.empty(N, H, d, dtype=torch.bfloat16, device=dev)
+                    ms = timed(lambda: qwm.qwm_attend(cfg, cache, qd[:N], kd[:N], vd[:N], out=out))
+                    fl = 2.0 * H * N * (L * (2 * d + r) + N * 2 * d)
+                    tf = fl / (ms * 1e-3) / 1e12
+                    attend_pts.append({"N": N, "L": L, "r": r, "ms": round(ms, 4), "tflops": round(tf, 1),
+                                       "frac_bf16": round(tf / pk["bf16_tflops"], 4)})
+        if cache.status():
+            raise RuntimeError("device status after the attend sweep")
+        del cache
+    append_pts = []
+    for N in Ns:
+        kN, vN = kd[:N].contiguous(), vd[:N].contiguous()
+        for C in Cs:
+            cfit = qwm.config(H, C, kmeans_iters=10)
+            kc = qwm.qwm_fit_centroids(cfit, kN)
+            vc = qwm.qwm_fit_centroids(cfit, vN)
+            for r in rs:
+                U = synth.population_U(a, r).to(dev) if r > 0 else None
+                for G in Gs:
+                    cfg = qwm.config(H, C, group_size=G, psac_rank=r, candidates=4)
+                    ring = qwm.Cache(cfg, N, 1, sliding_window=True, device=dev)
+                    ms = timed(lambda: qwm.qwm_quantize_append(cfg, ring, kN, vN, kc, vc, w=w, U=U))
+                    if ring.status():
+                        raise RuntimeError("device status after an append point")
+                    wlp = synth.Workload("p", heads=H, chunk_tokens=N, past_chunks=0, centroids=C, group_size=G,
+                                         psac_rank=r)
+                    nb = workload_numbers(wlp)["append_bytes"]
+                    gbs = nb / (ms * 1e-3) / 1e9
+                    append_pts.append({"N": N, "C": C, "r": r, "G": G, "ms": round(ms, 4), "gbs": round(gbs, 1),
+                                       "frac_hbm": round(gbs / pk["hbm_gbs"], 4)})
+                    del ring
+    return {"metric": "one-layer microbench sweep (40 heads): attend TFLOP/s and append GB/s per point",
+            "unit": "TFLOP/s | GB/s", "data": "synthetic", "dtype": "f16",
+            "peaks": {"bf16_tflops": pk["bf16_tflops"], "hbm_gbs": pk["hbm_gbs"], "src": pk["src"]},
+            "attend": attend_pts, "append": append_pts,
+            "l2": "256 MB flush before each timed call; median of %d" % reps}
+
+
 # ---------------------------------------------------------------------------- CPU oracle
 def cpu_model():
     """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
@@ -614,6 +833,10 @@ def main():
                     help="group scale storage: 0 binary16 per group, 1 uint8 codes + binary16 per token")
     ap.add_argument("--heads", type=int, default=0,
                     help="profiling only: the workload with fewer heads (same per-head work); not a bench line")
+    ap.add_argument("--psac-rank", type=int, default=-1,
+                    help="layer stacks: PSAC rank other than the workload's own (the 1.3B DiT at r = 32)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="the one-layer microbench sweep (N x L x C x r x G); prints one JSON object")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -624,6 +847,13 @@ def main():
         wl = dataclasses.replace(wl, heads=args.heads, name=f"{wl.name}_h{args.heads}")
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
+
+    if args.sweep and args.impl != "reference":
+        print(json.dumps(run_sweep(args)), flush=True)
+        return
+    if wl.layers > 1 and args.impl != "reference":
+        print(json.dumps(stack_line(args, wl, None if args.psac_rank < 0 else args.psac_rank)), flush=True)
+        return
 
     if args.impl == "reference":
         if rank != 0:
