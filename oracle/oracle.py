@@ -299,6 +299,29 @@ def top1_shift(idx_ref, idx):
 
 
 # ---------------------------------------------------------------- storage accounting
+def psac_tile_layout(kept, r: int, tile: int = 128):
+    """The App. D.1 choice between dense and sparse PSAC coefficient layouts,
+    made for each tile of `tile` tokens of a chunk-head (reading: the cache's
+    storage unit; the paper leaves the granularity and the index format open).
+    Dense stores every row's r INT8 codes and binary16 scale, n_t (r + 2)
+    bytes; sparse stores a keep bit per token of the tile (a tile/8-byte mask,
+    the index) and the kept rows only, tile/8 + K_t (r + 2) bytes, in token
+    order; the strictly smaller one is chosen.  kept: bool/uint8 [N].
+    Returns (sparse [ntiles] bool, bytes [ntiles] of the chosen layout)."""
+    kept = np.asarray(kept).astype(bool)
+    N = kept.size
+    nt = (N + tile - 1) // tile
+    sparse = np.zeros(nt, bool)
+    nbytes = np.zeros(nt, np.int64)
+    for t in range(nt):
+        k = kept[t * tile:(t + 1) * tile]
+        dense_b = k.size * (r + 2)
+        sparse_b = tile // 8 + int(k.sum()) * (r + 2)
+        sparse[t] = sparse_b < dense_b
+        nbytes[t] = min(dense_b, sparse_b)
+    return sparse, nbytes
+
+
 def psac_layout_bytes(kept, r: int, N: int | None = None):
     """Bytes of one chunk-head's PSAC coefficients in the two layouts App. D.1
     chooses between (reading: dense = every row's r INT8 codes and binary16

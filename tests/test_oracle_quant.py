@@ -444,6 +444,31 @@ def test_two_level_scales_zero_token_and_psac_layout(orc):
     assert orc.psac_layout_bytes(kept, 8) == (1000, 1204, 1000)
 
 
+def test_psac_tile_layout_hand_cases(orc):
+    """Per-tile layout choice (App. D.1, reading: dense n_t (r + 2) bytes,
+    sparse 16-byte keep mask + K_t (r + 2)): hand-counted boundary cases."""
+    k = np.zeros(128, bool)
+    k[:10] = True                                    # 10 kept of 128, r = 16
+    sp, nb = orc.psac_tile_layout(k, 16)
+    assert list(sp) == [True] and list(nb) == [16 + 10 * 18]
+    k[:] = True                                      # all kept: the mask only adds
+    assert orc.psac_tile_layout(k, 16)[0].tolist() == [False]
+    assert orc.psac_tile_layout(k, 16)[1].tolist() == [128 * 18]
+    k[5] = False                                     # 127 kept: 16 + 127*18 = 2302 < 2304
+    assert orc.psac_tile_layout(k, 16)[0].tolist() == [True]
+    assert orc.psac_tile_layout(k, 16)[1].tolist() == [2302]
+    assert orc.psac_tile_layout(k, 8)[0].tolist() == [False]   # r = 8: 16 + 127*10 = 1286 > 1280
+    k[6] = False                                                # 126 kept, r = 8: 1276 < 1280
+    assert orc.psac_tile_layout(k, 8)[1].tolist() == [1276]
+    # two tiles and a ragged tail of 72 tokens, all kept in the tail: dense there
+    k3 = np.zeros(328, bool)
+    k3[:64] = True
+    k3[256:] = True
+    sp, nb = orc.psac_tile_layout(k3, 16)
+    assert sp.tolist() == [True, True, False]
+    assert nb.tolist() == [16 + 64 * 18, 16, 72 * 18]
+
+
 
 # ------------------------------------------------------------------ full-matrix distance (App. C.4 ablation)
 def test_full_matrix_distance_reduces_to_diagonal_and_matches_fp64(orc):
