@@ -93,7 +93,15 @@ typedef struct qwm_cache qwm_cache;
  *     16+2i (App. D.1 packs four codes per byte; this order is ours);
  *   scales [128][d/G] binary16; ids [128] u8;
  *   zero-points [128][zb] u8: group g in byte g/4, bits 2(g%4);
- *   Keys only: PSAC codes [128][r] int8 and row scales [128] binary16.
+ *   Keys only: PSAC codes [128][r] int8 and row scales [128] binary16, in one
+ *     of two layouts per tile (App. D.1 stores the smaller of a dense and a
+ *     sparse coefficient layout): the tile's 16-byte keep mask at
+ *     pmask_offset + 16 * tile (bit i of the little-endian 128-bit mask = row
+ *     i) names the rows stored; row i's codes and scale are entry
+ *     e = popcount(mask bits below i) of the two arrays.  Dense tiles set a
+ *     bit for every token (rows whose correction was dropped hold zeros);
+ *     sparse tiles set the kept rows only, so they take 16 + K (r + 2) bytes
+ *     instead of n (r + 2), and are chosen when that is smaller.
  * With scale_format 1 the scale field holds [128][d/G] u8 codes and a
  * secondary scale field [128] binary16 follows it (k_s2, v_s2). */
 typedef struct qwm_layout {
@@ -108,6 +116,7 @@ typedef struct qwm_layout {
   int64_t zero_bytes;       /* zb: bytes of packed zero-points per token */
   int64_t k_s2, v_s2;       /* scale_format 1: secondary scales [128] binary16 (k_scales, v_scales
                                then hold [128][d/G] uint8 codes); 0 otherwise */
+  int64_t pmask_offset;     /* within a head: PSAC keep masks [tiles_per_chunk][16 B] (r > 0) */
 } qwm_layout;
 
 /* Human-readable name of a status code (static string). */
@@ -117,7 +126,7 @@ QWM_API const char* qwm_status_string(qwm_status status);
  * tokens needs (App. D.1 packed storage: per token-head d/4 code bytes, d/G
  * binary16 scales, one uint8 centroid id, 2-bit zero-points, for Keys r INT8
  * PSAC codes + one binary16 row scale; per chunk-head the two centroid
- * tables as binary16 and U_r^T as bf16).  Returns 0 for an invalid or
+ * tables as binary16, U_r^T as bf16 and a 16-byte PSAC keep mask per tile).  Returns 0 for an invalid or
  * unsupported configuration. */
 QWM_API size_t qwm_cache_bytes(const qwm_config* cfg, int64_t tokens_per_chunk, int32_t max_chunks);
 

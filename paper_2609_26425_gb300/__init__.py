@@ -63,7 +63,7 @@ class QwmLayout(ct.Structure):
         "ktab_offset", "vtab_offset", "ut_offset", "tiles_offset",
         "tile_tokens", "tiles_per_chunk", "tile_bytes",
         "k_codes", "k_scales", "k_ids", "k_zeros", "k_coef", "k_sigma", "k_bytes",
-        "v_codes", "v_scales", "v_ids", "v_zeros", "v_bytes", "zero_bytes", "k_s2", "v_s2")]
+        "v_codes", "v_scales", "v_ids", "v_zeros", "v_bytes", "zero_bytes", "k_s2", "v_s2", "pmask_offset")]
 
 
 _lib = None
@@ -221,7 +221,10 @@ class Cache:
         sigma [N][H] (binary16 bits), k_tab / v_tab [H][C][d] (binary16 bits,
         the tables as stored in the slot) and U [H][d][r] (bf16 bits).  With
         scale_format 1, scode [N][H][d/G] u8 and s2 [N][H] (binary16 bits)
-        replace scales (and v_scode, v_s2 for Values)."""
+        replace scales (and v_scode, v_s2 for Values).  PSAC rows are read
+        through each tile's keep mask (row i is entry popcount(mask below i);
+        rows the mask leaves out hold zeros) and returned per token; pmask
+        [H][tiles][4] u32 holds the masks as stored."""
         slot, N = self.chunk_info(i)
         lay = self.layout()
         cfg = self.cfg
@@ -238,6 +241,7 @@ class Cache:
         k_tab = np.zeros((H, C, d), np.uint16)
         v_tab = np.zeros((H, C, d), np.uint16)
         U = np.zeros((H, d, r), np.uint16)
+        pmask = np.zeros((H, ntile, 4), np.uint32)
         for h in range(H):
             hb = lay.slot_meta_bytes + h * lay.head_bytes
             k_tab[h] = raw[hb + lay.ktab_offset: hb + lay.ktab_offset + C * d * 2].view(np.uint16).reshape(C, d)
@@ -262,13 +266,27 @@ class Cache:
                 out["v_scales"].append(f(lay.v_scales, ng * 2, np.uint16))
             out["ids"].append(f(lay.k_ids, 1)[:, 0])
             out["zeros"].append(f(lay.k_zeros, zb))
-            out["coef"].append(f(lay.k_coef, r, np.int8) if r else np.zeros((N, 0), np.int8))
-            out["sigma"].append(f(lay.k_sigma, 2, np.uint16)[:, 0] if r else np.zeros(N, np.uint16))
+            if r:
+                pm = raw[hb + lay.pmask_offset: hb + lay.pmask_offset + ntile * 16].view(np.uint32).reshape(ntile, 4)
+                pmask[h] = pm
+                bitsel = ((pm[:, np.arange(T) // 32] >> (np.arange(T) % 32).astype(np.uint32)) & 1).astype(bool)
+                entry = np.cumsum(bitsel, axis=1) - 1
+                ct = np.ascontiguousarray(tiles[:, lay.k_coef: lay.k_coef + T * r]).view(np.int8).reshape(ntile, T, r)
+                st = np.ascontiguousarray(tiles[:, lay.k_sigma: lay.k_sigma + T * 2]).view(np.uint16).reshape(ntile, T)
+                tix = np.arange(ntile)[:, None]
+                e = np.where(bitsel, entry, 0)
+                cf = np.where(bitsel[..., None], ct[tix, e], 0).astype(np.int8).reshape(ntile * T, r)[:N]
+                sg = np.where(bitsel, st[tix, e], 0).astype(np.uint16).reshape(ntile * T)[:N]
+                out["coef"].append(cf)
+                out["sigma"].append(sg)
+            else:
+                out["coef"].append(np.zeros((N, 0), np.int8))
+                out["sigma"].append(np.zeros(N, np.uint16))
             out["v_codes"].append(f(lay.v_codes, d // 4))
             out["v_ids"].append(f(lay.v_ids, 1)[:, 0])
             out["v_zeros"].append(f(lay.v_zeros, zb))
         res = {k: np.stack(v, axis=1) for k, v in out.items()}
-        res.update(k_tab=k_tab, v_tab=v_tab, U=U, tokens=N, slot=slot)
+        res.update(k_tab=k_tab, v_tab=v_tab, U=U, tokens=N, slot=slot, pmask=pmask)
         return res
 
 

@@ -518,6 +518,7 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
   float* sW = reinterpret_cast<float*>(sm + S::W);
   float* sMisc = reinterpret_cast<float*>(sm + S::MISC);
   int* sRsCount = reinterpret_cast<int*>(sm + S::MISC + 64);
+  uint32_t* sPMask = reinterpret_cast<uint32_t*>(sm + S::MISC + 16);  // the tile's PSAC keep bits, per warp
   uint16_t* sRsPair = reinterpret_cast<uint16_t*>(sm + S::RS);
   float* sRsDq = reinterpret_cast<float*>(sm + S::RSD);
   const uint32_t bar = smem_u32(sm + S::BAR);
@@ -979,6 +980,11 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
     if (tid == 0 && u + 1 < u1) issue_tile(u + 1);
 
     // ---- part B: stores, PSAC
+    uint32_t pcw[R > 0 ? R / 4 : 1];  // this token's PSAC codes and row scale when kept (Keys)
+#pragma unroll
+    for (int i = 0; i < (R > 0 ? R / 4 : 1); ++i) pcw[i] = 0;
+    __half psg = __ushort_as_half(0);
+    bool pkept = false;
     if (valid) {
       reinterpret_cast<uint4*>(dcodes)[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
       reinterpret_cast<uint4*>(dcodes)[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
@@ -1007,12 +1013,6 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
       // the keep rule (Eq. 16), Keys only
       if constexpr (R > 0) {
         if (is_key) {
-          int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)tid * R);
-          __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma) + tid;
-          uint32_t cwd[R / 4];
-    #pragma unroll
-          for (int i = 0; i < R / 4; ++i) cwd[i] = 0;
-          __half sgh_out = __ushort_as_half(0);
           if (psac) {
             float c[R], v[R];
     #pragma unroll
@@ -1103,19 +1103,54 @@ __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
             }
             if (keep) {
     #pragma unroll
-              for (int i = 0; i < R / 4; ++i) cwd[i] = tq[i];
-              sgh_out = sgh;
+              for (int i = 0; i < R / 4; ++i) pcw[i] = tq[i];
+              psg = sgh;
+              pkept = true;
             }
           }
+        }
+      }
+    }
+
+    // ---- 6. the tile's PSAC rows in the smaller of the two layouts (App.
+    // D.1): dense (every token's row, dropped corrections as zeros) or
+    // sparse (only the kept rows, compacted in token order), with the tile's
+    // 128-bit keep mask naming the rows stored (row i is entry
+    // popcount(mask below i)).
+    if constexpr (R > 0) {
+      if (is_key) {
+        const uint32_t wm = __ballot_sync(0xFFFFFFFFu, pkept);
+        if (lane == 0) sPMask[warp] = wm;
+        __syncthreads();
+        uint32_t m4[4] = {sPMask[0], sPMask[1], sPMask[2], sPMask[3]};
+        const int nt = (int)((a.N - (int64_t)tile * 128) < 128 ? (a.N - (int64_t)tile * 128) : 128);
+        const int Kt = __popc(m4[0]) + __popc(m4[1]) + __popc(m4[2]) + __popc(m4[3]);
+        const bool sparse = 16 + Kt * (R + 2) < nt * (R + 2);
+        int e = tid;
+        if (sparse) {
+          e = __popc(m4[warp] & ((1u << lane) - 1u));
+#pragma unroll
+          for (int w4 = 0; w4 < 3; ++w4) e += w4 < warp ? __popc(m4[w4]) : 0;
+        } else {
+#pragma unroll
+          for (int w4 = 0; w4 < 4; ++w4) {
+            const int nb = nt - 32 * w4;
+            m4[w4] = nb >= 32 ? 0xFFFFFFFFu : (nb > 0 ? (1u << nb) - 1u : 0u);
+          }
+        }
+        if (valid && (!sparse || pkept)) {
+          int8_t* coef = reinterpret_cast<int8_t*>(tb + L.k_coef + (int64_t)e * R);
           if constexpr (R == 8) {
-            *reinterpret_cast<uint2*>(coef) = make_uint2(cwd[0], cwd[1]);
+            *reinterpret_cast<uint2*>(coef) = make_uint2(pcw[0], pcw[1]);
           } else {
     #pragma unroll
             for (int i = 0; i < R / 16; ++i)
-              reinterpret_cast<uint4*>(coef)[i] = make_uint4(cwd[4 * i], cwd[4 * i + 1], cwd[4 * i + 2], cwd[4 * i + 3]);
+              reinterpret_cast<uint4*>(coef)[i] = make_uint4(pcw[4 * i], pcw[4 * i + 1], pcw[4 * i + 2], pcw[4 * i + 3]);
           }
-          *sig = sgh_out;
+          reinterpret_cast<__half*>(tb + L.k_sigma)[e] = psg;
         }
+        if (tid == 0)
+          *reinterpret_cast<uint4*>(head + L.pmask + (int64_t)tile * 16) = make_uint4(m4[0], m4[1], m4[2], m4[3]);
       }
     }
   }

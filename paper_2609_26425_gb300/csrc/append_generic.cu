@@ -126,6 +126,19 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
   if (psac)
     for (int i = tid; i < 128 * r; i += NT) s.U[i] = a.U[(size_t)h * 128 * r + i];  // [d][r]
   if (nbad) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
+  // This kernel stores the dense PSAC layout: every token of a tile has its
+  // row (dropped corrections as zeros), so the tile's keep mask names all of
+  // them; the CTA holding a tile's first token writes it.
+  if (is_key && r > 0 && tid == 0 && t0 % kTile == 0) {
+    const int64_t nt64 = a.N - t0;
+    const int nt = (int)(nt64 < kTile ? nt64 : kTile);
+    uint32_t m4[4];
+    for (int w4 = 0; w4 < 4; ++w4) {
+      const int nb = nt - 32 * w4;
+      m4[w4] = nb >= 32 ? 0xFFFFFFFFu : (nb > 0 ? (1u << nb) - 1u : 0u);
+    }
+    *reinterpret_cast<uint4*>(head + L.pmask + (t0 / kTile) * 16) = make_uint4(m4[0], m4[1], m4[2], m4[3]);
+  }
   __syncthreads();
   if (tid < ng) {
     float Wg = 0.0f;

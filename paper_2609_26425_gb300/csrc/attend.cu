@@ -466,7 +466,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       }
       return v;
     };
+    // the tile's PSAC keep mask (which rows its code and scale arrays hold),
+    // loaded one tile ahead with the ids and used only in the next tile's
+    // passes, so no warp waits for it
+    auto load_pm = [&](const TileCursor& c) -> uint4 {
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (c.valid() && c.U.hb && c.U.psac && q * 8 < r) v = ldg16(c.U.hb + L.pmask + (int64_t)c.tl * 16);
+      return v;
+    };
     uint32_t idn = load_ids(cur);
+    uint4 pmn = load_pm(cur);
     uint32_t jt = 0;
     bool ok = true;
     const int kt = tid - 32 * 8;  // 0..127
@@ -475,6 +484,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         *reinterpret_cast<uint4*>(sm + OFF_U + 16 * idx) = make_uint4(0u, 0u, 0u, 0u);
     while (cur.valid()) {
       const uint32_t idc = idn;
+      const uint4 pmc = pmn;
       TileCursor nc = cur;
       nc.next(a, S, h);
       const int st = jt & 1;
@@ -500,6 +510,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           }
         }
         const bool psac_lane = cur.U.psac && q * 8 < r;
+        // entries of the lane's two rows in the tile's PSAC arrays (-1: none):
+        // the rows lie in this CTA's half of the tile (mask words 2c, 2c + 1),
+        // entry = kept rows below the row
+        int pe0 = -1, pe1 = -1;
+        if (psac_lane) {
+          const uint32_t lo = rank ? pmc.z : pmc.x, hi = rank ? pmc.w : pmc.y;
+          const int base = rank ? __popc(pmc.x) + __popc(pmc.y) : 0;
+          const int b0 = wrow & 31, b1 = (wrow + 8) & 31;
+          const uint32_t w0 = wrow >= 32 ? hi : lo, w1 = wrow + 8 >= 32 ? hi : lo;
+          const int o0 = base + (wrow >= 32 ? __popc(lo) : 0), o1 = base + (wrow + 8 >= 32 ? __popc(lo) : 0);
+          if ((w0 >> b0) & 1u) pe0 = o0 + __popc(w0 & ((1u << b0) - 1u));
+          if ((w1 >> b1) & 1u) pe1 = o1 + __popc(w1 & ((1u << b1) - 1u));
+        }
         // One row per pass (loads, then its reconstruction); the pass loop is
         // kept rolled so that the four roles' hot loops stay small enough for
         // the instruction caches.
@@ -535,8 +558,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
                 scv[1] = __half_as_ushort(__hmul(__uint2half_rn(__ldg(cp8 + ((64 + 16 * q) >> gshift))), s2));
               }
               if (psac_lane) {
-                cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)trw * r + q * 8));
-                sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + trw * 2));
+                // the tile's keep mask names the stored rows; row trw is entry e
+                const int e = p ? pe1 : pe0;
+                if (e >= 0) {
+                  cfv = __ldg(reinterpret_cast<const uint2*>(tb + L.k_coef + (int64_t)e * r + q * 8));
+                  sgv = __ldg(reinterpret_cast<const unsigned short*>(tb + L.k_sigma + e * 2));
+                }
               }
             } else {
               const __nv_bfloat16* src = a.kcur + ((size_t)(cur.tl * 128 + trw) * H + h) * 128;
@@ -596,6 +623,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
+      pmn = load_pm(nc);
       cur = nc;
       ++jt;
     }

@@ -47,9 +47,12 @@ __global__ void __launch_bounds__(256) dequant_kernel(const DequantArgs a) {
     float v[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) v[e] = __half2float(tab[c0 + e]) + s * (float)(qv[e] - z);
-    if (side == 0 && a.psac && L.r > 0) {
-      const float sg = __half2float(*reinterpret_cast<const __half*>(tb + L.k_sigma + row * 2));
-      const int8_t* t = reinterpret_cast<const int8_t*>(tb + L.k_coef + row * L.r);
+    const int pe = (side == 0 && a.psac && L.r > 0)
+                       ? psac_entry(*reinterpret_cast<const uint4*>(head + L.pmask + tile * 16), (int)row)
+                       : -1;
+    if (pe >= 0) {
+      const float sg = __half2float(*reinterpret_cast<const __half*>(tb + L.k_sigma + pe * 2));
+      const int8_t* t = reinterpret_cast<const int8_t*>(tb + L.k_coef + pe * L.r);
       const __nv_bfloat16* Ut = reinterpret_cast<const __nv_bfloat16*>(head + L.ut);  // [r][128]
       for (int j = 0; j < L.r; ++j) {
         const float cj = (float)t[j] * sg;

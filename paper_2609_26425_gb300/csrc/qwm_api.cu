@@ -200,6 +200,7 @@ qwm_status qwm_cache_layout(const qwm_cache* c, qwm_layout* o) {
   o->zero_bytes = L.zb;
   o->k_s2 = L.k_s2;
   o->v_s2 = L.v_s2;
+  o->pmask_offset = L.pmask;
   return QWM_OK;
 }
 

@@ -32,7 +32,7 @@ struct Layout {
   int64_t v_codes, v_scales, v_ids, v_zeros, v_bytes;  // from the tile start
   int64_t k_s2, v_s2;    // scale format 1: secondary scales [128] binary16
   int64_t tile_bytes;
-  int64_t ktab, vtab, ut, tiles_off, head_bytes;
+  int64_t ktab, vtab, ut, pmask, tiles_off, head_bytes;  // pmask: [tiles][16 B] PSAC keep masks (r > 0)
   int64_t slot_bytes;
   int64_t total_bytes;
 };
@@ -66,12 +66,25 @@ inline Layout make_layout(const qwm_config& c, int64_t T, int32_t max_chunks) {
   L.ktab = o;      o += (int64_t)L.C * L.d * 2;
   L.vtab = o;      o += (int64_t)L.C * L.d * 2;
   L.ut = o;        o += (int64_t)L.r * L.d * 2;
+  L.pmask = o;     o += L.r > 0 ? L.tiles * 16 : 0;
   o = round_up(o, 1024);
   L.tiles_off = o; o += L.tiles * L.tile_bytes;
   L.head_bytes = round_up(o, 1024);
   L.slot_bytes = kSlotMetaBytes + (int64_t)L.H * L.head_bytes;
   L.total_bytes = kHeaderBytes + (int64_t)max_chunks * L.slot_bytes;
   return L;
+}
+
+// Entry of row `row` (0..127) of a tile in its PSAC code and scale arrays, or
+// -1 when the tile's keep mask (4 little-endian words) does not name the row:
+// the entry is the number of mask bits below the row (App. D.1 dense/sparse
+// layouts; a dense tile names every row, so the entry is the row).
+__device__ __forceinline__ int psac_entry(uint4 m, int row) {
+  const int wi = row >> 5, bi = row & 31;
+  const uint32_t w = wi == 0 ? m.x : (wi == 1 ? m.y : (wi == 2 ? m.z : m.w));
+  if (!((w >> bi) & 1u)) return -1;
+  return __popc(w & ((1u << bi) - 1u)) + (wi > 0 ? __popc(m.x) : 0) + (wi > 1 ? __popc(m.y) : 0) +
+         (wi > 2 ? __popc(m.z) : 0);
 }
 
 __host__ __device__ inline int64_t head_offset(const Layout& L, int slot, int h) {

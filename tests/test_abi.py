@@ -39,8 +39,9 @@ def test_library_exports_every_declared_symbol(qlib):
 
 def test_cache_bytes_matches_packed_format(qlib):
     """Per token-head: d/4 code bytes, d/G binary16 scales, 1 id byte, the zero-point
-    byte; Keys add r INT8 codes + a binary16 row scale; per chunk-head two bf16
-    centroid tables and U_r^T.  Tiles hold 128 tokens."""
+    byte; Keys add r INT8 codes + a binary16 row scale; per chunk-head two
+    binary16 centroid tables, U_r^T and a 16-byte PSAC keep mask per tile.
+    Tiles hold 128 tokens."""
     for (H, C, G, r, T, n) in [(40, 256, 32, 16, 4680, 6), (4, 64, 32, 16, 880, 3), (12, 64, 64, 8, 880, 15),
                                (2, 16, 32, 0, 100, 1)]:
         cfg = qlib.config(H, C, group_size=G, psac_rank=r)
@@ -49,7 +50,7 @@ def test_cache_bytes_matches_packed_format(qlib):
         k_tok = d // 4 + 2 * ng + 1 + 1 + (r + 2 if r else 0)
         v_tok = d // 4 + 2 * ng + 1 + 1
         tiles = -(-T // 128)
-        per_head = 2 * C * d * 2 + r * d * 2
+        per_head = 2 * C * d * 2 + r * d * 2 + (16 * tiles if r else 0)   # + a PSAC keep mask per tile
         per_head = -(-per_head // 1024) * 1024 + tiles * 128 * (k_tok + v_tok)
         per_head = -(-per_head // 1024) * 1024
         assert b == 256 + n * (256 + H * per_head)
@@ -117,7 +118,7 @@ def test_cache_bytes_two_level_scales(qlib):
         k_tok = d // 4 + ng + 2 + 1 + 1 + (r + 2 if r else 0)
         v_tok = d // 4 + ng + 2 + 1 + 1
         tiles = -(-T // 128)
-        per_head = 2 * C * d * 2 + r * d * 2
+        per_head = 2 * C * d * 2 + r * d * 2 + (16 * tiles if r else 0)
         per_head = -(-per_head // 1024) * 1024 + tiles * 128 * (k_tok + v_tok)
         per_head = -(-per_head // 1024) * 1024
         assert b == 256 + n * (256 + H * per_head)

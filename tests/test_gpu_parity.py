@@ -107,6 +107,57 @@ def test_append_parity_two_level_scales(H, N, C, G, r, M):
     assert sk["id_flips"] <= max(1, N * H // 1000)
 
 
+@pytest.mark.parametrize("H,N,C,r,M,use_U", [
+    (2, 300, 64, 16, 4, True),       # the filter + quantize path, ragged tail tile
+    (2, 257, 16, 8, 4, True),        # r = 8: a tile needs two dropped rows to go sparse
+    (3, 130, 64, 32, 1, True),
+    (2, 200, 8, 16, 8, True),        # exhaustive QSAC (M = C)
+    (2, 300, 64, 16, 4, False),      # cold start: no row kept, every tile sparse and empty
+    (2, 150, 64, 16, 12, True),      # 8 < M < C: the exhaustive-distance kernel stores dense tiles
+])
+def test_psac_tile_layout_matches_oracle(H, N, C, r, M, use_U):
+    """App. D.1 dense/sparse PSAC layouts per 128-token tile: the GPU stores
+    the layout the oracle chooses (keep mask, byte count), and the rows read
+    back through the mask equal the oracle's (compare_packed)."""
+    _, k, v = make_chunk(H * 77 + N, N, H)
+    kb, vb = synth.bits(k), synth.bits(v)
+    kc, vc = strided_centroids(kb, C), strided_centroids(vb, C)
+    w = synth.random_weights(N + 5, H, 128).numpy()
+    Ub = synth.bits(synth.random_orthonormal(N + 6, H, 128, r)) if use_U else None
+    cfg = qwm.config(H, C, psac_rank=r, candidates=M)
+    cache = qwm.Cache(cfg, N, 1)
+    qwm.qwm_quantize_append(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
+                            w=torch.from_numpy(w).cuda(), U=None if Ub is None else dev(synth.from_bits(Ub)))
+    assert cache.status() == 0
+    dec = cache.decode_chunk(0)
+    ko, vo = oracle_append(kb, vb, kc, vc, G=32, r=r, M=M, w=w, U_bits=Ub)
+    compare_packed(dec, ko, kb, kc, G=32, r=r, M=M, is_key=True, w=w, U_bits=Ub)
+    ntile = -(-N // 128)
+    for h in range(H):
+        pm = dec["pmask"][h]
+        full = np.zeros((ntile, 4), np.uint32)
+        for t in range(ntile):
+            nt = min(128, N - 128 * t)
+            for wd in range(4):
+                nb = nt - 32 * wd
+                full[t, wd] = 0xFFFFFFFF if nb >= 32 else ((1 << nb) - 1 if nb > 0 else 0)
+        gpu_sparse = (pm != full).any(-1)
+        kept_bits = np.array([[bin(int(x)).count("1") for x in row] for row in pm]).sum(-1)
+        sp, nb = orc.psac_tile_layout(ko["kept"][:, h], r)
+        if 8 < M < C:
+            assert not gpu_sparse.any()
+            continue
+        assert np.array_equal(gpu_sparse, sp), (h, gpu_sparse, sp)
+        gpu_bytes = np.where(gpu_sparse, 16 + kept_bits * (r + 2),
+                             np.minimum(128, N - 128 * np.arange(ntile)) * (r + 2))
+        assert np.array_equal(gpu_bytes, nb)
+        # a sparse tile's mask is the oracle's keep set
+        for t in np.nonzero(sp)[0]:
+            kt = ko["kept"][128 * t: 128 * t + 128, h].astype(bool)
+            bits = ((pm[t][np.arange(kt.size) // 32] >> (np.arange(kt.size) % 32).astype(np.uint32)) & 1).astype(bool)
+            assert np.array_equal(bits, kt)
+
+
 def test_append_parity_fitted_tables():
     """Tables from the oracle's k-means (the realistic case: many near ties)."""
     run_append_case(4, 880, 64, 32, 16, 4, True, True, seed=7, fit_iters=10)
