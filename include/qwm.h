@@ -229,6 +229,20 @@ QWM_API qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* cache, 
                                int64_t N, const void* k_centroids, const void* v_centroids,
                                const float* w, const void* U, void* stream);
 
+/* qwm_quantize_append with the Keys' top-M candidates chosen by the full
+ * Query-aware quadratic form d_j = (k - mu_j)^T M (k - mu_j) instead of its
+ * diagonal (Eq. 9): the ablation of App. C.4 (the QSAC score and everything
+ * after still use w; Values unchanged).  Mq: fp32 [H][d][d] row-major, the
+ * historical Query second moment of each head (Eq. 6) or any symmetric
+ * matrix, 16-byte aligned.  As in the oracle, d_j is the fp32 evaluation
+ * e = k - mu_j, t_c = sum_c' M_cc' e_c' and d = sum_c e_c t_c, one fused
+ * multiply-add per term in index order; the tensor cores screen the
+ * candidates (B operand M mu_j) and the undecided rows are rescored with it.
+ * 8 < num_candidates < num_centroids returns QWM_ERR_UNSUPPORTED. */
+QWM_API qwm_status qwm_quantize_append_full(const qwm_config* cfg, qwm_cache* cache, const void* k, const void* v,
+                                            int64_t N, const void* k_centroids, const void* v_centroids,
+                                            const float* w, const void* U, const float* Mq, void* stream);
+
 /* Attention of Nq new queries over every cached chunk and the active chunk
  * (Sec. 3.3 Eq. 5 logits; Sec. 4.2 Eq. 17: Q K_hat^T = Q K_hat0^T +
  * (Q U_r) C^T with each chunk's own U_r; Values rebuilt without PSAC).

@@ -120,6 +120,8 @@ def lib():
             L.qwm_dequant_chunk.restype = ct.c_int
             L.qwm_top1_keys.argtypes = [_CFG, _P, ct.c_int64, _P, ct.c_int64, _P, _P]
             L.qwm_top1_keys.restype = ct.c_int
+            L.qwm_quantize_append_full.argtypes = [_CFG, _P, _P, _P, ct.c_int64, _P, _P, _P, _P, _P, _P]
+            L.qwm_quantize_append_full.restype = ct.c_int
             L.qwm_cache_set_wait_limit.argtypes = [_P, ct.c_uint64]
             L.qwm_cache_set_wait_limit.restype = ct.c_int
             L.qwm_cache_set_idle_role.argtypes = [_P, ct.c_int32]
@@ -338,6 +340,27 @@ def qwm_quantize_append(cfg: QwmConfig, cache: Cache, k, v, k_centroids, v_centr
     _check("qwm_quantize_append", lib().qwm_quantize_append(
         ct.byref(cfg), cache.handle, _ptr(k), _ptr(v), N, _ptr(k_centroids), _ptr(v_centroids), _ptr(w),
         _ptr(U), _stream()))
+
+
+def qwm_quantize_append_full(cfg: QwmConfig, cache: Cache, k, v, k_centroids, v_centroids, Mq, w=None, U=None):
+    """qwm_quantize_append with the Keys' candidates by the full quadratic form
+    (Mq: fp32 CUDA tensor [H][d][d])."""
+    N = k.shape[0]
+    H, d, C, r = cfg.num_heads, cfg.head_dim, cfg.num_centroids, cfg.psac_rank
+    _bf16(k, (N, H, d), "k")
+    _bf16(v, (N, H, d), "v")
+    _bf16(k_centroids, (H, C, d), "k_centroids")
+    _bf16(v_centroids, (H, C, d), "v_centroids")
+    if not (Mq.is_cuda and Mq.dtype == torch.float32 and Mq.is_contiguous() and tuple(Mq.shape) == (H, d, d)):
+        raise ValueError("Mq must be a contiguous fp32 CUDA tensor [H][d][d]")
+    if w is not None:
+        if not (w.is_cuda and w.dtype == torch.float32 and w.is_contiguous() and tuple(w.shape) == (H, d)):
+            raise ValueError("w must be a contiguous fp32 CUDA tensor [H][d]")
+    if U is not None:
+        _bf16(U, (H, d, r), "U")
+    _check("qwm_quantize_append_full", lib().qwm_quantize_append_full(
+        ct.byref(cfg), cache.handle, _ptr(k), _ptr(v), N, _ptr(k_centroids), _ptr(v_centroids), _ptr(w),
+        _ptr(U), _ptr(Mq), _stream()))
 
 
 def qwm_attend(cfg: QwmConfig, cache: Cache, q, k_cur=None, v_cur=None, sm_scale=None, out=None,

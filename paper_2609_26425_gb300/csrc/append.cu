@@ -47,9 +47,6 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kMaxFilterM = 8;
-constexpr int kBand = 16;         // band members listed for exact rescoring
-constexpr int kRecAll = 255;      // record: rescore every centroid
 
 __device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
 __device__ __forceinline__ uint4 lds16(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
@@ -101,8 +98,8 @@ constexpr int F_BLO = 65536;
 constexpr int F_A = 131072;                 // FG x [2][128 rows][128 B]
 constexpr int F_AJ = F_A + FG * 32768;      // A_j [256] fp32
 constexpr int F_W = F_AJ + 1024;            // w [128]
-constexpr int F_RED = F_W + 512;            // [8 warps][2]
-constexpr int F_LIST = F_RED + 64;          // FNT x 32-byte records
+constexpr int F_RED = F_W + 512;            // [8 warps][4]
+constexpr int F_LIST = F_RED + 128;         // FNT x 32-byte records
 constexpr int F_BAR = F_LIST + FNT * 32;    // 4 mbarriers, flags, TMEM slot
 constexpr int F_SMEM = F_BAR + 64 + 1024;
 
@@ -167,8 +164,81 @@ __global__ void __launch_bounds__(FNT, 1)
     // ---- B_hi, B_lo and A_j of this (head, side)
     if (tid < 128) sW[tid] = use_w ? a.w[(size_t)h * 128 + tid] : 1.0f;
     __syncthreads();
-    float n2 = 0.0f, amax = 0.0f;
-    {
+    // With the full quadratic form (App. C.4, Keys only), B = M mu_j and
+    // A_j = mu_j^T M mu_j; the bound then needs max |mu_j| and the largest
+    // row sum of |M| (mun2, mabs).
+    const bool full = is_key && a.Mq != nullptr;
+    const float* Mh = full ? a.Mq + (size_t)h * 128 * 128 : nullptr;
+    float n2 = 0.0f, amax = 0.0f, mun2 = 0.0f, mabs = 0.0f;
+    if (full && tid < 128) {
+      const float4* Mr = reinterpret_cast<const float4*>(Mh + (size_t)tid * 128);
+      for (int c4 = 0; c4 < 32; ++c4) {
+        const float4 m4 = __ldg(Mr + c4);
+        mabs += fabsf(m4.x) + fabsf(m4.y) + fabsf(m4.z) + fabsf(m4.w);
+      }
+      mabs *= 1.0001f;  // the fp32 sum of the absolute values, rounded up
+    }
+    if (full) {
+      const int j = tid;
+      if (j < C) {
+        const __nv_bfloat16* mr = tab + (size_t)j * 128;
+        uint32_t muw[64];
+#pragma unroll
+        for (int ch = 0; ch < 16; ++ch) {
+          const uint4 m = ldg16(mr + ch * 8);
+          muw[4 * ch] = m.x; muw[4 * ch + 1] = m.y; muw[4 * ch + 2] = m.z; muw[4 * ch + 3] = m.w;
+        }
+        float A = 0.0f;
+#pragma unroll 1
+        for (int ch = 0; ch < 16; ++ch) {
+          float b8[8];
+#pragma unroll
+          for (int o = 0; o < 8; ++o) {
+            const float4* Mr = reinterpret_cast<const float4*>(Mh + (size_t)(ch * 8 + o) * 128);
+            float acc = 0.0f;
+#pragma unroll
+            for (int c4 = 0; c4 < 32; ++c4) {
+              const float4 m4 = __ldg(Mr + c4);
+              const uint32_t w0 = muw[2 * c4], w1 = muw[2 * c4 + 1];
+              acc = fmaf(m4.x, __uint_as_float(w0 << 16), acc);
+              acc = fmaf(m4.y, __uint_as_float(w0 & 0xFFFF0000u), acc);
+              acc = fmaf(m4.z, __uint_as_float(w1 << 16), acc);
+              acc = fmaf(m4.w, __uint_as_float(w1 & 0xFFFF0000u), acc);
+            }
+            b8[o] = acc;
+          }
+          uint32_t hw[4], lw[4];
+#pragma unroll
+          for (int p2 = 0; p2 < 4; ++p2) {
+            const float b0 = b8[2 * p2], b1 = b8[2 * p2 + 1];
+            const uint32_t mw = muw[4 * ch + p2];
+            const float m0 = __uint_as_float(mw << 16), m1 = __uint_as_float(mw & 0xFFFF0000u);
+            A = fmaf(m0, b0, fmaf(m1, b1, A));
+            n2 = fmaf(b0, b0, fmaf(b1, b1, n2));
+            mun2 = fmaf(m0, m0, fmaf(m1, m1, mun2));
+            const __half2 hh = __floats2half2_rn(b0, b1);
+            const float2 hf = __half22float2(hh);
+            hw[p2] = *reinterpret_cast<const uint32_t*>(&hh);
+            lw[p2] = pack_f16(b0 - hf.x, b1 - hf.y);
+          }
+          const int off = sw_off(Npad, j, ch);
+          *reinterpret_cast<uint4*>(sm + F_BHI + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+          *reinterpret_cast<uint4*>(sm + F_BLO + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        }
+        sAj[j] = A;
+        amax = fabsf(A);
+      } else {
+        if (j < Npad) {
+#pragma unroll
+          for (int ch = 0; ch < 16; ++ch) {
+            const int off = sw_off(Npad, j, ch);
+            *reinterpret_cast<uint4*>(sm + F_BHI + off) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(sm + F_BLO + off) = make_uint4(0, 0, 0, 0);
+          }
+        }
+        sAj[j] = INFINITY;  // j in [C, 256): never selected
+      }
+    } else {
       const int j = tid;
       if (j < C) {
         const __nv_bfloat16* mr = tab + (size_t)j * 128;
@@ -211,20 +281,27 @@ __global__ void __launch_bounds__(FNT, 1)
     for (int off = 16; off; off >>= 1) {
       n2 = fmaxf(n2, __shfl_xor_sync(0xFFFFFFFFu, n2, off));
       amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, off));
+      mun2 = fmaxf(mun2, __shfl_xor_sync(0xFFFFFFFFu, mun2, off));
+      mabs = fmaxf(mabs, __shfl_xor_sync(0xFFFFFFFFu, mabs, off));
     }
     if (lane == 0) {
-      sRed[2 * warp] = n2;
-      sRed[2 * warp + 1] = amax;
+      sRed[4 * warp] = n2;
+      sRed[4 * warp + 1] = amax;
+      sRed[4 * warp + 2] = mun2;
+      sRed[4 * warp + 3] = mabs;
     }
     fence_proxy_async_smem();
     __syncthreads();
-    float W2 = 0.0f, Am = 0.0f;
+    float W2 = 0.0f, Am = 0.0f, Mu2 = 0.0f, Mab = 0.0f;
 #pragma unroll
     for (int i = 0; i < FNT / 32; ++i) {
-      W2 = fmaxf(W2, sRed[2 * i]);
-      Am = fmaxf(Am, sRed[2 * i + 1]);
+      W2 = fmaxf(W2, sRed[4 * i]);
+      Am = fmaxf(Am, sRed[4 * i + 1]);
+      Mu2 = fmaxf(Mu2, sRed[4 * i + 2]);
+      Mab = fmaxf(Mab, sRed[4 * i + 3]);
     }
     const float Wn = sqrtf(W2);
+    const float Mun = sqrtf(Mu2) * 1.0001f;
 
     // ---- the tiles of this run, alternating between the two groups
     for (int u = s0 + g; u < s1; u += FG) {
@@ -372,7 +449,11 @@ __global__ void __launch_bounds__(FNT, 1)
 
       const float kth = sel_at(tv, Mc - 1), nxt = sel_at(tv, Mc);
       const float kn = sqrtf(kn2);
-      const float Bb = ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
+      // full quadratic form: every candidate's oracle value and ours lie within
+      // 2^-13 (|k| + max|mu|)^2 max_c sum_c' |M_cc'| of the exact form (the
+      // oracle's own sequential fp32 rounding is the larger part)
+      const float Bb = full ? ldexpf((kn + Mun) * (kn + Mun) * Mab, -13) + 1e-30f
+                            : ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
       const float lim = kth + 2.0f * Bb;
       // a list overflow (more than kList columns at or below T), a row out of
       // the binary16 range, or a table whose w o mu rows reach beyond it (the
@@ -1204,6 +1285,10 @@ cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
     kern<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    if (a.Mq) {  // the Keys' undecided rows, rescored with the full quadratic form
+      e = launch_full_rescore(a, st);
+      if (e != cudaSuccess) return e;
+    }
   }
   switch (a.L.r) {
     case 0: return launch_quant_r<0>(a, tk, tv, st);

@@ -237,9 +237,11 @@ qwm_status qwm_fit_centroids(const qwm_config* cfg, const void* x, int64_t N, vo
   return qwm::launch_fit(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
 }
 
-qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* c, const void* k, const void* v, int64_t N,
-                               const void* k_centroids, const void* v_centroids, const float* w, const void* U,
-                               void* stream) {
+namespace {
+
+qwm_status quantize_append(const qwm_config* cfg, qwm_cache* c, const void* k, const void* v, int64_t N,
+                           const void* k_centroids, const void* v_centroids, const float* w, const void* U,
+                           const float* Mq, void* stream) {
   if (!cfg || !c || !k || !v || !k_centroids || !v_centroids) return QWM_ERR_INVALID_ARG;
   if (!supported(cfg)) return QWM_ERR_UNSUPPORTED;
   if (!same_shape(cfg, &c->cfg)) return QWM_ERR_INVALID_ARG;
@@ -264,11 +266,30 @@ qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* c, const void* 
   a.w = w;
   a.U = (cfg->psac_rank > 0) ? static_cast<const __nv_bfloat16*>(U) : nullptr;
   a.M = cfg->num_candidates < cfg->num_centroids ? cfg->num_candidates : cfg->num_centroids;
+  a.Mq = Mq;
   if (qwm::launch_append(a, static_cast<cudaStream_t>(stream)) != cudaSuccess) return QWM_ERR_CUDA;
   c->n_tokens[slot] = (int32_t)N;
   c->psac[slot] = a.U != nullptr;
   c->appended += 1;
   return QWM_OK;
+}
+
+}  // namespace
+
+qwm_status qwm_quantize_append(const qwm_config* cfg, qwm_cache* c, const void* k, const void* v, int64_t N,
+                               const void* k_centroids, const void* v_centroids, const float* w, const void* U,
+                               void* stream) {
+  return quantize_append(cfg, c, k, v, N, k_centroids, v_centroids, w, U, nullptr, stream);
+}
+
+qwm_status qwm_quantize_append_full(const qwm_config* cfg, qwm_cache* c, const void* k, const void* v, int64_t N,
+                                    const void* k_centroids, const void* v_centroids, const float* w, const void* U,
+                                    const float* Mq, void* stream) {
+  if (!Mq || !aligned16(Mq)) return QWM_ERR_INVALID_ARG;
+  if (!cfg) return QWM_ERR_INVALID_ARG;
+  // the exhaustive-distance kernel of 8 < M < C takes the diagonal form only
+  if (cfg->num_candidates > 8 && cfg->num_candidates < cfg->num_centroids) return QWM_ERR_UNSUPPORTED;
+  return quantize_append(cfg, c, k, v, N, k_centroids, v_centroids, w, U, Mq, stream);
 }
 
 qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, int64_t Nq, const void* k_cur,

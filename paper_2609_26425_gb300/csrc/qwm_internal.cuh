@@ -119,9 +119,19 @@ struct AppendArgs {
   const float* w;              // [H][d] or null
   const __nv_bfloat16* U;      // [H][d][r] or null
   int M;                       // candidates (clamped to C)
+  const float* Mq;             // [H][d][d] fp32: Keys' candidates by the full quadratic form, or null
 };
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
 cudaError_t launch_append_generic(const AppendArgs& a, cudaStream_t s);
+cudaError_t launch_full_rescore(const AppendArgs& a, cudaStream_t s);
+
+// The candidate filter's per-token record, parked in the token's 32 code
+// bytes of the destination slot until the quantize kernel reads it: byte 0 =
+// n, bytes 1.. = centroid ids.  n = M: the decided top-M; M <= n <= kBand:
+// the band to rescore exactly; kRecAll: rescore every centroid.
+constexpr int kMaxFilterM = 8;
+constexpr int kBand = 16;
+constexpr int kRecAll = 255;
 
 struct AttendSlots {
   int32_t n;

@@ -158,6 +158,59 @@ def test_psac_tile_layout_matches_oracle(H, N, C, r, M, use_U):
             assert np.array_equal(bits, kt)
 
 
+@pytest.mark.parametrize("kind,H,N,C,M", [
+    ("diag", 2, 300, 64, 4),       # M = diag(w): the full form evaluated on a diagonal matrix
+    ("dense", 2, 300, 64, 4),      # a dense symmetric positive M
+    ("dense", 2, 257, 256, 2),     # the largest table, ragged tile
+    ("dense", 1, 130, 16, 1),
+    ("dense", 2, 200, 8, 8),       # M = C: every centroid a candidate (the matrix plays no part)
+])
+def test_append_full_matrix_distance_parity(kind, H, N, C, M):
+    """App. C.4 ablation: the Keys' top-M candidates by the full quadratic form
+    (k - mu)^T M (k - mu), bit-exact against the oracle's full-form path
+    under the margin rule (the QSAC score and everything after keep w)."""
+    _, k, v = make_chunk(H * 31 + N, N, H)
+    kb, vb = synth.bits(k), synth.bits(v)
+    kc, vc = strided_centroids(kb, C), strided_centroids(vb, C)
+    w = synth.random_weights(N + 11, H, 128).numpy()
+    r = 16
+    Ub = synth.bits(synth.random_orthonormal(N + 12, H, 128, r))
+    if kind == "diag":
+        Mq = np.stack([np.diag(w[h]) for h in range(H)]).astype(np.float32)
+    else:
+        R = np.random.default_rng(N).standard_normal((H, 128, 128))
+        Mq = (np.einsum("hij,hkj->hik", R, R) / 128).astype(np.float32)
+    cfg = qwm.config(H, C, psac_rank=r, candidates=M)
+    cache = qwm.Cache(cfg, N, 1)
+    qwm.qwm_quantize_append_full(cfg, cache, dev(k), dev(v), dev(synth.from_bits(kc)), dev(synth.from_bits(vc)),
+                                 torch.from_numpy(Mq).cuda(), w=torch.from_numpy(w).cuda(), U=dev(synth.from_bits(Ub)))
+    assert cache.status() == 0
+    dec = cache.decode_chunk(0)
+    ko = orc.quantize(kb, kc, G=32, r=r, M=M, is_key=True, w=w, U_bits=Ub, M_full=Mq)
+    vo = orc.quantize(vb, vc, G=32, r=r, M=M, is_key=False)
+    # margin-rule requantisation keeps the full form: compare ids through the oracle with M_full
+    diff = dec["ids"] != ko["ids"]
+    if diff.any():
+        margin = np.minimum(ko["m_topm"], ko["m_sel"])
+        assert not (diff & (margin >= 1e-5)).any()
+        ko = orc.quantize(kb, kc, G=32, r=r, M=M, is_key=True, w=w, U_bits=Ub, M_full=Mq, force_ids=dec["ids"])
+    for key in ("codes", "scales", "zeros"):
+        assert np.array_equal(dec[key], ko[key]), key
+    row_bad = (dec["coef"] != ko["coef"]).any(-1) | (dec["sigma"] != ko["sigma"])
+    assert np.all(ko["m_psac"][row_bad] < 1e-5)
+    compare_packed(dec, vo, vb, vc, G=32, r=r, M=M, is_key=False, prefix="v_")
+
+
+def test_append_full_matrix_rejects_the_exhaustive_kernel_range():
+    cfg = qwm.config(2, 64, candidates=12)
+    cache = qwm.Cache(cfg, 10, 1)
+    z = torch.zeros(10, 2, 128, dtype=torch.bfloat16, device="cuda")
+    t = torch.zeros(2, 64, 128, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(qwm.QwmError) as e:
+        qwm.qwm_quantize_append_full(cfg, cache, z, z, t, t, torch.zeros(2, 128, 128, device="cuda"))
+    assert e.value.status == 2
+
+
 def test_append_parity_fitted_tables():
     """Tables from the oracle's k-means (the realistic case: many near ties)."""
     run_append_case(4, 880, 64, 32, 16, 4, True, True, seed=7, fit_iters=10)
