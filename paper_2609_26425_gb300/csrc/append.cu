@@ -104,8 +104,9 @@ constexpr int F_BAR = F_LIST + FNT * 32;    // 4 mbarriers, flags, TMEM slot
 constexpr int F_SMEM = F_BAR + 64 + 1024;
 
 // CAPT = M + 1 (the ranked list of a row), or kMaxFilterM + 1 for the
-// candidate counts without their own instance.
-template <int CAPT>
+// candidate counts without their own instance; FULL: the Keys' distance is
+// the full quadratic form (qwm_quantize_append_full).
+template <int CAPT, bool FULL>
 __global__ void __launch_bounds__(FNT, 1)
     append_filter(const AppendArgs a, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, int tiles, int units) {
@@ -167,7 +168,7 @@ __global__ void __launch_bounds__(FNT, 1)
     // With the full quadratic form (App. C.4, Keys only), B = M mu_j and
     // A_j = mu_j^T M mu_j; the bound then needs max |mu_j| and the largest
     // row sum of |M| (mun2, mabs).
-    const bool full = is_key && a.Mq != nullptr;
+    const bool full = FULL && is_key;
     const float* Mh = full ? a.Mq + (size_t)h * 128 * 128 : nullptr;
     float n2 = 0.0f, amax = 0.0f, mun2 = 0.0f, mabs = 0.0f;
     if (full && tid < 128) {
@@ -1275,8 +1276,10 @@ cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    auto kern = a.M == 4 ? append_filter<5> : (a.M == 1 ? append_filter<2> : (a.M == 2 ? append_filter<3>
-                                                                                      : append_filter<kMaxFilterM + 1>));
+    auto kern = a.Mq ? (a.M == 4 ? append_filter<5, true> : (a.M == 1 ? append_filter<2, true>
+                                     : (a.M == 2 ? append_filter<3, true> : append_filter<kMaxFilterM + 1, true>)))
+                     : (a.M == 4 ? append_filter<5, false> : (a.M == 1 ? append_filter<2, false>
+                                     : (a.M == 2 ? append_filter<3, false> : append_filter<kMaxFilterM + 1, false>)));
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
     if (e != cudaSuccess) return e;
     const int tiles = (int)((a.N + 127) / 128);
