@@ -52,9 +52,10 @@ def workload_numbers(wl, scale_format=0):
             "k_bytes_per_token_head": k_tok, "v_bytes_per_token_head": v_tok}
 
 
-def attend_traffic():
+def attend_traffic(workload):
     """DRAM bytes per attend launch from the committed ncu summary, or None when
-    the kernel source has changed since those counters were taken."""
+    the kernel source has changed since those counters were taken or the
+    workload is not the one they were taken on."""
     import hashlib
     prof = os.path.join(ROOT, "profiles", "attend_kernel_wan14b_layer.md")
     src = os.path.join(ROOT, "paper_2609_26425_gb300", "csrc", "attend.cu")
@@ -62,12 +63,12 @@ def attend_traffic():
         fields = {}
         with open(prof) as f:
             for line in f:
-                if ":" in line and line.split(":")[0] in ("traffic_bytes_per_launch", "source_sha256"):
+                if ":" in line and line.split(":")[0] in ("traffic_bytes_per_launch", "source_sha256", "workload"):
                     k, v = line.split(":", 1)
                     fields[k.strip()] = v.strip()
         with open(src, "rb") as f:
             digest = hashlib.sha256(f.read()).hexdigest()
-        if fields.get("source_sha256") == digest:
+        if fields.get("source_sha256") == digest and fields.get("workload") == workload:
             return int(fields["traffic_bytes_per_launch"])
     except (OSError, ValueError, KeyError):
         pass
@@ -341,7 +342,7 @@ def run_gpu(args, wl, rank, world):
                    "algorithmic_bytes": nums["append_bytes"]},
         "roofline": {"bound": "tensor", "kernel": "attend_kernel", "achieved": round(att_tflops, 2),
                      "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                     "frac": round(att_tflops / pk["bf16_tflops"], 4), "traffic": attend_traffic(),
+                     "frac": round(att_tflops / pk["bf16_tflops"], 4), "traffic": attend_traffic(None if args.scale_format else wl.name),
                      "peak_src": pk["src"] + " burst bf16 (binary16 operands run at the bf16 rate)"},
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         # attend: one kernel; append: the candidate filter and the quantize kernel

@@ -450,11 +450,18 @@ __global__ void __launch_bounds__(FNT, 1)
 
       const float kth = sel_at(tv, Mc - 1), nxt = sel_at(tv, Mc);
       const float kn = sqrtf(kn2);
-      // full quadratic form: every candidate's oracle value and ours lie within
-      // 2^-13 (|k| + max|mu|)^2 max_c sum_c' |M_cc'| of the exact form (the
-      // oracle's own sequential fp32 rounding is the larger part)
-      const float Bb = full ? ldexpf((kn + Mun) * (kn + Mun) * Mab, -13) + 1e-30f
-                            : ldexpf(kn * Wn + Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) + 1e-30f;
+      // |our dt_j - the oracle's d_j + common term| <= Bb for every candidate.
+      // The tensor cores' fp32 accumulation is taken to move the sum by at most
+      // two ulps of its running absolute value per product added (256 products:
+      // 2^-14 |k| |B_j| by Cauchy-Schwarz, twice that in dt = A - 2 D); the
+      // operand split adds 2^-22 |k| |B_j|, the fp32 A_j and the oracle's
+      // sequential sums 2^-17 of their magnitudes each, and binary16 subnormal
+      // operands an absolute 2^-25 per element (the 2^-19 term).  For the full
+      // form (App. C.4) every one of these is below 2^-13 (|k| + max|mu|)^2
+      // max_c sum_c' |M_cc'| (the norm of M for a symmetric M).
+      const float Bb = full ? ldexpf((kn + Mun) * (kn + Mun) * Mab, -13) + ldexpf(kn + Wn, -19) + 1e-30f
+                            : ldexpf(kn * Wn, -13) + ldexpf(Am + K0 + fabsf(kth), -16) + ldexpf(kn + Wn, -19) +
+                                  1e-30f;
       const float lim = kth + 2.0f * Bb;
       // a list overflow (more than kList columns at or below T), a row out of
       // the binary16 range, or a table whose w o mu rows reach beyond it (the
