@@ -126,19 +126,9 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
   if (psac)
     for (int i = tid; i < 128 * r; i += NT) s.U[i] = a.U[(size_t)h * 128 * r + i];  // [d][r]
   if (nbad) atomicCAS(reinterpret_cast<int*>(a.base), 0, (int)QWM_ERR_NONFINITE);
-  // This kernel stores the dense PSAC layout: every token of a tile has its
-  // row (dropped corrections as zeros), so the tile's keep mask names all of
-  // them; the CTA holding a tile's first token writes it.
-  if (is_key && r > 0 && tid == 0 && t0 % kTile == 0) {
-    const int64_t nt64 = a.N - t0;
-    const int nt = (int)(nt64 < kTile ? nt64 : kTile);
-    uint32_t m4[4];
-    for (int w4 = 0; w4 < 4; ++w4) {
-      const int nb = nt - 32 * w4;
-      m4[w4] = nb >= 32 ? 0xFFFFFFFFu : (nb > 0 ? (1u << nb) - 1u : 0u);
-    }
-    *reinterpret_cast<uint4*>(head + L.pmask + (t0 / kTile) * 16) = make_uint4(m4[0], m4[1], m4[2], m4[3]);
-  }
+  // PSAC rows are written at their token's index; each kept row sets its bit
+  // in the tile's keep mask (zeroed before the launch), and psac_tile_finish
+  // then stores each tile in the dense or the sparse layout.
   __syncthreads();
   if (tid < ng) {
     float Wg = 0.0f;
@@ -389,9 +379,57 @@ __global__ void __launch_bounds__(NT, 1) append_generic_kernel(const AppendArgs 
         keep = __shfl_sync(0xFFFFFFFFu, keep, 0);
         if (lane < r) coef[lane] = (int8_t)(keep ? tq : 0);
         if (lane == 0) *sig = keep ? sgh : __ushort_as_half(0);
+        if (lane == 0 && keep)
+          atomicOr(reinterpret_cast<unsigned int*>(head + L.pmask + tile * 16) + (rowi >> 5), 1u << (rowi & 31));
       }
     }
     __syncwarp();
+  }
+}
+
+// The dense/sparse PSAC layout of each 128-token Key tile (App. D.1), from the
+// keep mask the quantize kernel left: with n_t tokens and K_t kept rows the
+// tile is sparse iff 16 + K_t (r + 2) < n_t (r + 2) (a 16-byte mask plus the
+// kept rows against every row).  Dense: the mask becomes the tile's full
+// token mask (dropped rows already hold zeros).  Sparse: the mask stays the
+// keep set and kept row i moves to entry popcount(mask below i), through
+// shared memory (the moves overlap in place).  One CTA per (tile, head),
+// thread = row.
+__global__ void __launch_bounds__(kTile) psac_tile_finish(const AppendArgs a) {
+  __shared__ uint2 srow[kTile][4];  // up to 32 code bytes per row
+  __shared__ __half ssig[kTile];
+  const Layout& L = a.L;
+  const int tile = blockIdx.x, h = blockIdx.y, i = threadIdx.x, r = L.r;
+  uint8_t* head = a.base + head_offset(L, a.slot, h);
+  uint4* mp = reinterpret_cast<uint4*>(head + L.pmask + (int64_t)tile * 16);
+  const uint4 m = *mp;
+  const int64_t nt64 = a.N - (int64_t)tile * kTile;
+  const int nt = nt64 < kTile ? (int)nt64 : kTile;
+  const int K = __popc(m.x) + __popc(m.y) + __popc(m.z) + __popc(m.w);
+  if (!(16 + K * (r + 2) < nt * (r + 2))) {
+    if (i == 0) {
+      uint32_t m4[4];
+      for (int w4 = 0; w4 < 4; ++w4) {
+        const int nb = nt - 32 * w4;
+        m4[w4] = nb >= 32 ? 0xFFFFFFFFu : (nb > 0 ? (1u << nb) - 1u : 0u);
+      }
+      *mp = make_uint4(m4[0], m4[1], m4[2], m4[3]);
+    }
+    return;
+  }
+  uint8_t* tb = head + L.tiles_off + (int64_t)tile * L.tile_bytes;
+  uint2* coef = reinterpret_cast<uint2*>(tb + L.k_coef);  // rows of r / 8 words
+  __half* sig = reinterpret_cast<__half*>(tb + L.k_sigma);
+  const int rw = r / 8;
+  const int e = i < nt ? psac_entry(m, i) : -1;
+  if (e >= 0) {
+    for (int q = 0; q < rw; ++q) srow[i][q] = coef[i * rw + q];
+    ssig[i] = sig[i];
+  }
+  __syncthreads();
+  if (e >= 0) {
+    for (int q = 0; q < rw; ++q) coef[e * rw + q] = srow[i][q];
+    sig[e] = ssig[i];
   }
 }
 
@@ -401,8 +439,17 @@ cudaError_t launch_append_generic(const AppendArgs& a, cudaStream_t st) {
   const size_t smem = smem_bytes(a.L.C, a.L.r);
   cudaError_t e = cudaFuncSetAttribute(append_generic_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
+  const int tiles = (int)((a.N + kTile - 1) / kTile);
+  if (a.L.r > 0) {  // the keep masks of this slot's heads start empty
+    e = cudaMemset2DAsync(a.base + head_offset(a.L, a.slot, 0) + a.L.pmask, (size_t)a.L.head_bytes, 0,
+                          (size_t)tiles * 16, (size_t)a.L.H, st);
+    if (e != cudaSuccess) return e;
+  }
   dim3 grid((unsigned)((a.N + TT - 1) / TT), (unsigned)a.L.H, 2);
   append_generic_kernel<<<grid, NT, smem, st>>>(a);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || a.L.r == 0) return e;
+  psac_tile_finish<<<dim3((unsigned)tiles, (unsigned)a.L.H), kTile, 0, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -113,7 +113,9 @@ def test_append_parity_two_level_scales(H, N, C, G, r, M):
     (3, 130, 64, 32, 1, True),
     (2, 200, 8, 16, 8, True),        # exhaustive QSAC (M = C)
     (2, 300, 64, 16, 4, False),      # cold start: no row kept, every tile sparse and empty
-    (2, 150, 64, 16, 12, True),      # 8 < M < C: the exhaustive-distance kernel stores dense tiles
+    (2, 150, 64, 16, 12, True),      # 8 < M < C: the exhaustive-distance kernel and its tile finish
+    (2, 150, 64, 16, 12, False),     # the same, cold start: every tile sparse and empty
+    (1, 333, 32, 32, 10, True),      # the same, r = 32, ragged tail tile
 ])
 def test_psac_tile_layout_matches_oracle(H, N, C, r, M, use_U):
     """App. D.1 dense/sparse PSAC layouts per 128-token tile: the GPU stores
@@ -144,9 +146,6 @@ def test_psac_tile_layout_matches_oracle(H, N, C, r, M, use_U):
         gpu_sparse = (pm != full).any(-1)
         kept_bits = np.array([[bin(int(x)).count("1") for x in row] for row in pm]).sum(-1)
         sp, nb = orc.psac_tile_layout(ko["kept"][:, h], r)
-        if 8 < M < C:
-            assert not gpu_sparse.any()
-            continue
         assert np.array_equal(gpu_sparse, sp), (h, gpu_sparse, sp)
         gpu_bytes = np.where(gpu_sparse, 16 + kept_bits * (r + 2),
                              np.minimum(128, N - 128 * np.arange(ntile)) * (r + 2))
