@@ -16,7 +16,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libqwm.so")
-SOURCES = ["qwm_api.cu", "append.cu", "append_generic.cu", "append_full.cu", "attend.cu", "fit.cu", "qstats.cu",
+SOURCES = ["qwm_api.cu", "append.cu", "append_fused.cu", "append_fused_r8.cu", "append_fused_r16.cu",
+           "append_fused_r32.cu", "append_generic.cu", "append_full.cu", "attend.cu", "fit.cu", "qstats.cu",
            "metrics.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",

@@ -41,52 +41,13 @@
 // the generic kernel (append_generic.cu).
 #include "ptx_sm103.cuh"
 #include "qwm_internal.cuh"
+#include "append_common.cuh"
 
 namespace qwm {
 namespace {
 
 using namespace ptx;
 
-
-__device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
-__device__ __forceinline__ uint4 lds16(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
-// 32-byte read-only global load (address 32-byte aligned): one whole sector.
-__device__ __forceinline__ void ldg32(const void* p, uint32_t (&r)[8]) {
-  asm volatile("ld.global.nc.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-               : "l"(p));
-}
-
-// Byte offset of 16-byte chunk `ch` (channels 8ch..8ch+7) of row `row` in a
-// pair of 128-byte-swizzled blocks of `rows` rows x 64 two-byte elements.
-__device__ __forceinline__ int sw_off(int rows, int row, int ch) {
-  return (ch >> 3) * rows * 128 + row * 128 + (((ch & 7) ^ (row & 7)) << 4);
-}
-
-// Insert (v, j) into the ascending list of the n smallest (value, index)
-// pairs; indices arrive in ascending order, so an equal value stays behind.
-template <int CAP>
-__device__ __forceinline__ void insert_top(float (&tv)[CAP], int (&tj)[CAP], int n, float v, int j) {
-#pragma unroll
-  for (int s = 0; s < CAP; ++s) {
-    if (s < n && v < tv[s]) {
-      const float ov = tv[s];
-      const int oj = tj[s];
-      tv[s] = v;
-      tj[s] = j;
-      v = ov;
-      j = oj;
-    }
-  }
-}
-template <int CAP>
-__device__ __forceinline__ float sel_at(const float (&tv)[CAP], int i) {
-  float k = tv[0];
-#pragma unroll
-  for (int s = 1; s < CAP; ++s)
-    if (s == i) k = tv[s];
-  return k;
-}
 
 // ============================================================================
 // Kernel 1: candidate filter
@@ -556,8 +517,6 @@ struct QSmem {
 };
 
 constexpr int kRsCap = 512;             // (token, centroid) pairs rescored together per tile
-constexpr float kMagic = 12582912.0f;   // 1.5 * 2^23: (y + kMagic) - kMagic = rint(y) for |y| < 2^22
-constexpr float kTwo23 = 8388608.0f;
 
 // Exact Query-aware distance (Eq. 9) in channel order, one fused
 // multiply-add per term on the rounded square.
@@ -582,9 +541,6 @@ __device__ __forceinline__ float exact_dq(const uint8_t* sK, int row, const __nv
   return acc;
 }
 
-__device__ __forceinline__ float sel4(const float (&a)[4], int g) {
-  return g == 0 ? a[0] : (g == 1 ? a[1] : (g == 2 ? a[2] : a[3]));
-}
 
 template <int R, int GS>
 __global__ void __launch_bounds__(QNT, (R > 16 ? 3 : 4))
@@ -1275,31 +1231,28 @@ cudaError_t launch_quant_r(const AppendArgs& a, const CUtensorMap& tk, const CUt
 
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
   if (a.M > kMaxFilterM && a.M < a.L.C) return launch_append_generic(a, st);
+  if (!a.Mq || a.M >= a.L.C) return launch_append_fused(a, st);
+  // The Keys' candidates by the full quadratic form (App. C.4): the filter,
+  // the rescoring of its undecided rows, then the quantize kernel.
   alignas(64) CUtensorMap tk, tv;
   if (!make_token_map(&tk, a.k, a.N, a.L.H, 128) || !make_token_map(&tv, a.v, a.N, a.L.H, 128))
     return cudaErrorInvalidValue;
-  if (a.M < a.L.C) {
-    int dev = 0, nsm = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    auto kern = a.Mq ? (a.M == 4 ? append_filter<5, true> : (a.M == 1 ? append_filter<2, true>
-                                     : (a.M == 2 ? append_filter<3, true> : append_filter<kMaxFilterM + 1, true>)))
-                     : (a.M == 4 ? append_filter<5, false> : (a.M == 1 ? append_filter<2, false>
-                                     : (a.M == 2 ? append_filter<3, false> : append_filter<kMaxFilterM + 1, false>)));
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
-    if (e != cudaSuccess) return e;
-    const int tiles = (int)((a.N + 127) / 128);
-    const int units = 2 * a.L.H * tiles;
-    const int grid = units < nsm ? units : nsm;
-    kern<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    if (a.Mq) {  // the Keys' undecided rows, rescored with the full quadratic form
-      e = launch_full_rescore(a, st);
-      if (e != cudaSuccess) return e;
-    }
-  }
+  int dev = 0, nsm = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  auto kern = a.M == 4 ? append_filter<5, true> : (a.M == 1 ? append_filter<2, true>
+                  : (a.M == 2 ? append_filter<3, true> : append_filter<kMaxFilterM + 1, true>));
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, F_SMEM);
+  if (e != cudaSuccess) return e;
+  const int tiles = (int)((a.N + 127) / 128);
+  const int units = 2 * a.L.H * tiles;
+  const int grid = units < nsm ? units : nsm;
+  kern<<<grid, FNT, F_SMEM, st>>>(a, tk, tv, tiles, units);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  e = launch_full_rescore(a, st);
+  if (e != cudaSuccess) return e;
   switch (a.L.r) {
     case 0: return launch_quant_r<0>(a, tk, tv, st);
     case 8: return launch_quant_r<8>(a, tk, tv, st);

@@ -1,0 +1,11 @@
+// append_fused_r32.cu -- the fused append kernel (append_fused.cuh) for PSAC
+// rank 32, in a translation unit of its own so the ranks compile in parallel.
+#include "append_fused.cuh"
+
+namespace qwm {
+
+cudaError_t append_fused_r32(const AppendArgs& a, const CUtensorMap* maps, cudaStream_t st) {
+  return launch_fused_rank<32>(a, maps, st);
+}
+
+}  // namespace qwm

@@ -115,6 +115,21 @@ __device__ __forceinline__ bool named_bar_and(int id, int count, bool pred) {
   return r != 0;
 }
 
+// Named barrier over `count` threads that also returns the OR of their
+// predicates.
+__device__ __forceinline__ bool named_bar_or(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
+}
+
 // ----------------------------------------------------------------- packed fp32
 // Two fp32 lanes in one 64-bit register; every operation rounds each lane to
 // nearest even exactly as the scalar instruction would.

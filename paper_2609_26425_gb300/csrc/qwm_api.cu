@@ -36,6 +36,18 @@ bool make_token_map(CUtensorMap* m, const void* x, int64_t N, int H, int box_row
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool make_table_map(CUtensorMap* m, const void* tab, int C, int H, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn || C < 1 || H < 1 || box_rows < 1 || box_rows > 256) return false;
+  cuuint64_t dims[3] = {128, (cuuint64_t)C, (cuuint64_t)H};
+  cuuint64_t strides[2] = {256, (cuuint64_t)C * 256};
+  cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tab), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool make_row_map(CUtensorMap* m, const void* base, int64_t rows) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (!fn || rows < 1) return false;

@@ -103,6 +103,9 @@ bool make_token_map(CUtensorMap* m, const void* x, int64_t N, int H, int box_row
 // The cache buffer as rows of 256 bytes (128 binary16 values): boxes of 64
 // values x 1 row, 128-byte swizzle, for tile::gather4 loads of centroid rows.
 bool make_row_map(CUtensorMap* m, const void* base, int64_t rows);
+// Centroid tables tab[H][C][128] (bf16): boxes of 64 channels x box_rows
+// centroids x 1 head, 128-byte swizzle; rows past C read as zeros.
+bool make_table_map(CUtensorMap* m, const void* tab, int C, int H, int box_rows);
 
 // ----------------------------------------------------------------------------
 // Kernel launch entry points (defined in the .cu files).
@@ -123,6 +126,7 @@ struct AppendArgs {
 };
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t s);
 cudaError_t launch_append_generic(const AppendArgs& a, cudaStream_t s);
+cudaError_t launch_append_fused(const AppendArgs& a, cudaStream_t s);
 cudaError_t launch_full_rescore(const AppendArgs& a, cudaStream_t s);
 
 // The candidate filter's per-token record, parked in the token's 32 code
