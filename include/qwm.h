@@ -262,6 +262,27 @@ QWM_API qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* cache, con
                       const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,
                       void* out, float* lse, void* stream);
 
+/* Bytes of the scratch buffer that lets qwm_attend_ws balance a launch over
+ * the GPU (0: the launch needs none), for Nq queries over the cache's current
+ * chunks and N_cur active tokens on the current device; 0 for invalid
+ * arguments.  Not part of the paper's method: the launch's CTA pairs work on
+ * 512 queries of one head each, and when their count leaves the last wave of
+ * the SMs partly idle, the work units of that wave are split along the keys
+ * (whole chunks per part, cached chunks then the active chunk) and their
+ * partial results combined -- the usual rescaling of partial softmax sums,
+ * as for attention over several key blocks. */
+QWM_API size_t qwm_attend_workspace_bytes(const qwm_config* cfg, const qwm_cache* cache, int64_t Nq, int64_t N_cur);
+
+/* qwm_attend with a caller-owned device scratch buffer (256-byte aligned) of
+ * at least qwm_attend_workspace_bytes bytes for the same arguments: the same
+ * result within the attention tolerance (the parts of a split unit are
+ * combined in fp32; the bf16 output and the lse may differ from
+ * qwm_attend's in the last bits).  workspace = NULL, or a buffer too small,
+ * runs qwm_attend.  Calls sharing a buffer must not overlap on the GPU. */
+QWM_API qwm_status qwm_attend_ws(const qwm_config* cfg, const qwm_cache* cache, const void* q, int64_t Nq,
+                                 const void* k_cur, const void* v_cur, int64_t N_cur, float sm_scale,
+                                 void* out, float* lse, void* workspace, size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Historical Query statistics and the principal Query basis, kept on the GPU
  * (Sec. 4.1 Eq. 6 and 8, Sec. 4.2 Eq. 15; App. C.3 cold start; App. D.1: the

@@ -106,6 +106,11 @@ def lib():
             L.qwm_quantize_append.restype = ct.c_int
             L.qwm_attend.argtypes = [_CFG, _P, _P, ct.c_int64, _P, _P, ct.c_int64, ct.c_float, _P, _P, _P]
             L.qwm_attend.restype = ct.c_int
+            L.qwm_attend_workspace_bytes.argtypes = [_CFG, _P, ct.c_int64, ct.c_int64]
+            L.qwm_attend_workspace_bytes.restype = ct.c_size_t
+            L.qwm_attend_ws.argtypes = [_CFG, _P, _P, ct.c_int64, _P, _P, ct.c_int64, ct.c_float, _P, _P, _P,
+                                        ct.c_size_t, _P]
+            L.qwm_attend_ws.restype = ct.c_int
             L.qwm_query_stats_bytes.argtypes = [_CFG]
             L.qwm_query_stats_bytes.restype = ct.c_size_t
             L.qwm_query_stats_reset.argtypes = [_CFG, _P, _P]
@@ -363,8 +368,24 @@ def qwm_quantize_append_full(cfg: QwmConfig, cache: Cache, k, v, k_centroids, v_
         _ptr(U), _ptr(Mq), _stream()))
 
 
+def qwm_attend_workspace_bytes(cfg: QwmConfig, cache: Cache, Nq: int, Ncur: int = 0) -> int:
+    """Bytes of the scratch buffer qwm_attend can use to balance a launch (0: none needed)."""
+    return int(lib().qwm_attend_workspace_bytes(ct.byref(cfg), cache.handle, int(Nq), int(Ncur)))
+
+
+def attend_workspace(cfg: QwmConfig, cache: Cache, Nq: int, Ncur: int = 0, device=None):
+    """A torch-allocated scratch buffer for qwm_attend(..., workspace=), or None when none is needed."""
+    n = qwm_attend_workspace_bytes(cfg, cache, Nq, Ncur)
+    if n == 0:
+        return None
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    raw = torch.empty(n + 256, dtype=torch.uint8, device=dev)
+    off = (-raw.data_ptr()) % 256
+    return raw[off:off + n]
+
+
 def qwm_attend(cfg: QwmConfig, cache: Cache, q, k_cur=None, v_cur=None, sm_scale=None, out=None,
-               lse=None, want_lse=False):
+               lse=None, want_lse=False, workspace=None):
     Nq = q.shape[0]
     H, d = cfg.num_heads, cfg.head_dim
     _bf16(q, (Nq, H, d), "q")
@@ -378,9 +399,15 @@ def qwm_attend(cfg: QwmConfig, cache: Cache, q, k_cur=None, v_cur=None, sm_scale
     if want_lse and lse is None:
         lse = torch.empty(H, Nq, dtype=torch.float32, device=q.device)
     scale = 1.0 / math.sqrt(d) if sm_scale is None else float(sm_scale)
-    _check("qwm_attend", lib().qwm_attend(ct.byref(cfg), cache.handle, _ptr(q), Nq,
-                                          _ptr(k_cur) if Ncur else None, _ptr(v_cur) if Ncur else None, Ncur,
-                                          scale, _ptr(out), _ptr(lse), _stream()))
+    if workspace is None:
+        _check("qwm_attend", lib().qwm_attend(ct.byref(cfg), cache.handle, _ptr(q), Nq,
+                                              _ptr(k_cur) if Ncur else None, _ptr(v_cur) if Ncur else None, Ncur,
+                                              scale, _ptr(out), _ptr(lse), _stream()))
+    else:
+        _check("qwm_attend_ws", lib().qwm_attend_ws(ct.byref(cfg), cache.handle, _ptr(q), Nq,
+                                                    _ptr(k_cur) if Ncur else None, _ptr(v_cur) if Ncur else None,
+                                                    Ncur, scale, _ptr(out), _ptr(lse), _ptr(workspace),
+                                                    workspace.numel() * workspace.element_size(), _stream()))
     return (out, lse) if (want_lse or lse is not None) else out
 
 

@@ -149,9 +149,10 @@ __device__ __forceinline__ Unit unit_at(const AttendArgs& a, const AttendSlots& 
 struct TileCursor {
   int u, tl, n_units, ntiles;
   Unit U;
-  __device__ __forceinline__ void init(const AttendArgs& a, const AttendSlots& S, int h, int nu) {
-    u = 0; tl = 0; n_units = nu; ntiles = 0;
-    if (nu > 0) { U = unit_at(a, S, 0, h); ntiles = (U.ntok + 127) / 128; }
+  // the units [u0, u_end) (a part's range of chunks)
+  __device__ __forceinline__ void init(const AttendArgs& a, const AttendSlots& S, int h, int u0, int u_end) {
+    u = u0; tl = 0; n_units = u_end; ntiles = 0;
+    if (u0 < u_end) { U = unit_at(a, S, u0, h); ntiles = (U.ntok + 127) / 128; }
   }
   __device__ __forceinline__ bool valid() const { return u < n_units; }
   __device__ __forceinline__ void next(const AttendArgs& a, const AttendSlots& S, int h) {
@@ -189,21 +190,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const Layout& L = a.L;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  // Grid: x = 2 * (block of 512 queries) + rank (the CTA pair of a cluster),
-  // y = head (the pairs of one head run close together and share its packed
-  // tiles through L2).
-  const int h = blockIdx.y;
+  // Grid: x = 2 * (pair index) + rank (the CTA pair of a cluster).  Pair
+  // index P < n_whole is the work unit P = h * (blocks of 512 queries per
+  // head) + block, over every key; the later pairs are the parts of the tail
+  // units, each over a contiguous range of the key units (cached chunks, then
+  // the active chunk), whose partial results a second kernel combines.  The
+  // pairs of one head run close together and share its packed tiles through L2.
+  const int P = blockIdx.x >> 1;
+  const bool whole = P < a.n_whole;
+  const int wunit = whole ? P : a.n_whole + (P - a.n_whole) / a.nparts;
+  const int part = whole ? 0 : (P - a.n_whole) % a.nparts;
+  const int h = wunit / a.bph;
   const int H = L.H, r = L.r;
   const int rpad = r == 8 ? 16 : r;
   const int gshift = L.G == 32 ? 5 : 6;
   const uint32_t rank = cluster_rank();  // 0: leader
-  const int64_t pair0 = (int64_t)(blockIdx.x >> 1) * 512;
+  const int64_t pair0 = (int64_t)(wunit - h * a.bph) * 512;
   const int64_t q0 = pair0 + 256 * rank;
   // Q tiles the pair runs: the second is left out when neither CTA has a
   // query in it (the tail of the query range), halving that pair's MMA and
   // softmax work.
   const int nqt = pair0 + 128 < a.Nq ? 2 : 1;
-  const int n_units = S.n + (a.Ncur > 0 ? 1 : 0);
+  const int n_all = S.n + (a.Ncur > 0 ? 1 : 0);
+  // this pair's key units [cu0, cu1)
+  const int cu0 = whole ? 0 : (int)((int64_t)part * n_all / a.nparts);
+  const int cu1 = whole ? n_all : (int)((int64_t)(part + 1) * n_all / a.nparts);
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + OFF_BAR + NBAR * 8);
@@ -302,8 +313,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     float m_run = -INFINITY, l_run = 0.0f;
     uint32_t jt = 0;
     bool ok = true;
-    if (n_units > 0 && unit_at(a, S, 0, h).psac) ok = take_qu();
-    for (int u = 0; u < n_units && ok; ++u) {
+    if (cu0 < cu1 && unit_at(a, S, cu0, h).psac) ok = take_qu();
+    for (int u = cu0; u < cu1 && ok; ++u) {
       const Unit U = unit_at(a, S, u, h);
       const int ntiles = (U.ntok + 127) / 128;
       for (int tl = 0; tl < ntiles; ++tl, ++jt) {
@@ -396,10 +407,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         ok = handoff(B_PFULL + i, 1 + i, okw);
         if (!ok) break;
       }
-      if (ok && u + 1 < n_units && unit_at(a, S, u + 1, h).psac) ok = take_qu();
+      if (ok && u + 1 < cu1 && unit_at(a, S, u + 1, h).psac) ok = take_qu();
     }
     if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFINAL), 0, a.wait_ns));
-    if (ok) {
+    if (ok && (int)(blockIdx.x >> 1) < a.n_whole) {  // (recomputed: nothing kept live across the loop)
       tc_fence_after();
       const float inv_l = 1.0f / l_run;
       float v[32];
@@ -417,15 +428,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
       }
       if (a.lse && qvalid) a.lse[(size_t)h * a.Nq + qi] = m_run * a.sm_scale + logf(l_run);
+    } else if (ok) {
+      // a part of a tail unit: the unnormalised O row, the running maximum and
+      // sum, for the combining kernel
+      tc_fence_after();
+      const size_t prow = ((size_t)((int)(blockIdx.x >> 1) - a.n_whole) * 512 + 256 * rank + 128 * i + row);
+      float v[32];
+#pragma unroll
+      for (int cb = 0; cb < 4; ++cb) {
+        tmem_ld32(tO + cb * 32, v);
+        if (qvalid) {
+          float4* dst = reinterpret_cast<float4*>(a.part_o + prow * 128 + cb * 32);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+        }
+      }
+      if (qvalid) *reinterpret_cast<float2*>(a.part_ml + prow * 2) = make_float2(m_run, l_run);
     } else {
       *s_err = 1;
     }
     // Off the critical path: this CTA's share of the active chunk's rows of
     // head h (the rebuild converts them with saturation) is checked for values
     // beyond the binary16 range, which only the status word reports.
-    if (a.Ncur > 0) {
-      const int64_t per = (a.Ncur + gridDim.x - 1) / gridDim.x;
-      const int64_t r0 = (int64_t)blockIdx.x * per, r1 = min(a.Ncur, r0 + per);
+    const int P2 = (int)(blockIdx.x >> 1);
+    if (a.Ncur > 0 && (P2 < a.n_whole || (P2 - a.n_whole) % a.nparts == 0)) {
+      const int64_t gx = 2 * (int64_t)a.bph, bx = 2 * (pair0 >> 9) + rank;
+      const int64_t per = (a.Ncur + gx - 1) / gx;
+      const int64_t r0 = bx * per, r1 = min(a.Ncur, r0 + per);
       uint32_t mag = 0u;
       for (int64_t e = r0 * 16 + (tid & 255); e < r1 * 16; e += 256) {
         const int64_t tok = e >> 4;
@@ -451,7 +480,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     const int wrow = (warp & 3) * 16 + rr;  // local row of pass p: wrow + 8p
     const int tro = 64 * (int)rank;         // tile row of local row 0
     TileCursor cur;
-    cur.init(a, S, h, n_units);
+    cur.init(a, S, h, cu0, cu1);
     auto load_ids = [&](const TileCursor& c) -> uint32_t {  // 2 ids | 2 zero bytes << 16
       uint32_t v = 0;
       if (c.valid() && c.U.hb) {
@@ -640,7 +669,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     TileCursor cur;
     // an idle V role (the test hook of qwm_cache_set_idle_role) publishes no
     // tile: the MMA warp's bounded wait for the first one runs out
-    cur.init(a, S, h, a.idle_role == QWM_ROLE_V_REBUILD ? 0 : n_units);
+    cur.init(a, S, h, cu0, a.idle_role == QWM_ROLE_V_REBUILD ? cu0 : cu1);
     auto load_ids = [&](const TileCursor& c) -> uint64_t {  // 4 ids | 4 zero bytes << 32
       uint64_t v = 0;
       if (c.valid() && c.U.hb) {
@@ -745,16 +774,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       constexpr uint32_t idQU = idesc_f16(256, 64, false);
       constexpr uint32_t idPV = idesc_f16(256, 128, true);
       int total = 0;
-      for (int u = 0; u < n_units; ++u) total += (unit_at(a, S, u, h).ntok + 127) / 128;
+      for (int u = cu0; u < cu1; ++u) total += (unit_at(a, S, u, h).ntok + 127) / 128;
       TileCursor sc;  // next tile to issue S for
-      sc.init(a, S, h, n_units);
+      sc.init(a, S, h, cu0, cu1);
       uint32_t sjt = 0, qph[2] = {0, 0};
       bool ok = true;
       auto issue_S = [&](int i) -> bool {
         const int st = sjt & 1;
         const uint32_t ph = (sjt >> 1) & 1;
         if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph, a.wait_ns)) return false;
-        if (sc.tl == 0 && sc.u == 0) {  // Q_i in place
+        if (sc.tl == 0 && sc.u == cu0) {  // Q_i in place
           if (!mbar_wait_cluster(bar(B_QU + i), qph[i], a.wait_ns)) return false;
           qph[i] ^= 1;
         }
@@ -832,16 +861,85 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   }
 }
 
+
+// The parts of a tail unit combined (the usual rescaling of partial softmax
+// results: m = max_p m_p, l = sum_p l_p 2^((m_p - m) c), O = sum_p O_p
+// 2^((m_p - m) c) / l with c = sm_scale log2(e)); a warp per query row, four
+// channels per lane.
+__global__ void __launch_bounds__(256) attend_combine(const AttendArgs a) {
+  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // (tail unit, row)
+  const int lane = threadIdx.x & 31;
+  const int ntail = (a.n_units - a.n_whole);
+  if (gw >= (int64_t)ntail * 512) return;
+  const int tu = (int)(gw >> 9), prow = (int)(gw & 511);
+  const int unit = a.n_whole + tu;
+  const int h = unit / a.bph;
+  const int64_t qi = (int64_t)(unit - h * a.bph) * 512 + prow;
+  if (qi >= a.Nq) return;
+  const float c = a.sm_scale * 1.4426950408889634f;
+  float m = -INFINITY;
+  for (int p = 0; p < a.nparts; ++p) m = fmaxf(m, a.part_ml[((size_t)(tu * a.nparts + p) * 512 + prow) * 2]);
+  float l = 0.0f;
+  float4 o = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  for (int p = 0; p < a.nparts; ++p) {
+    const size_t pr = (size_t)(tu * a.nparts + p) * 512 + prow;
+    const float2 ml = *reinterpret_cast<const float2*>(a.part_ml + pr * 2);
+    const float wgt = exp2f((ml.x - m) * c);
+    l = fmaf(ml.y, wgt, l);
+    const float4 v = *reinterpret_cast<const float4*>(a.part_o + pr * 128 + 4 * lane);
+    o.x = fmaf(v.x, wgt, o.x); o.y = fmaf(v.y, wgt, o.y); o.z = fmaf(v.z, wgt, o.z); o.w = fmaf(v.w, wgt, o.w);
+  }
+  const float inv_l = 1.0f / l;
+  uint2* dst = reinterpret_cast<uint2*>(a.out + ((size_t)qi * a.L.H + h) * 128 + 4 * lane);
+  *dst = make_uint2(pack_bf16(o.x * inv_l, o.y * inv_l), pack_bf16(o.z * inv_l, o.w * inv_l));
+  if (a.lse && lane == 0) a.lse[(size_t)h * a.Nq + qi] = m * a.sm_scale + logf(l);
+}
+
 }  // namespace
+
+AttendPlan plan_attend(int64_t Nq, int H, int n_key_units, int nsm, bool split) {
+  AttendPlan pl{};
+  pl.bph = (int)((Nq + 511) / 512);
+  pl.n_units = pl.bph * H;
+  pl.n_whole = pl.n_units;
+  pl.nparts = 1;
+  const int slots = nsm / 2 > 0 ? nsm / 2 : 1;
+  if (!split || n_key_units < 2 || pl.n_units % slots == 0) return pl;
+  const int whole = pl.n_units / slots * slots, tail = pl.n_units - whole;
+  // parts per tail unit: the fewest rounds of the tail over the pair slots
+  // times the largest part (in key units), each part charged a fixed 0.15 of
+  // a key unit; ties to fewer parts
+  int best = 1;
+  double best_cost = (double)n_key_units + 0.15;
+  for (int s = 2; s <= n_key_units; ++s) {
+    const int rounds = (tail * s + slots - 1) / slots;
+    const int largest = (n_key_units + s - 1) / s;
+    const double cost = rounds * (largest + 0.15);
+    if (cost < best_cost - 1e-9) { best_cost = cost; best = s; }
+  }
+  if (best > 1) {
+    pl.n_whole = whole;
+    pl.nparts = best;
+  }
+  return pl;
+}
+
+size_t attend_workspace_bytes(const AttendPlan& pl) {
+  if (pl.nparts <= 1) return 0;
+  return (size_t)(pl.n_units - pl.n_whole) * pl.nparts * 512 * (128 + 2) * sizeof(float);
+}
 
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t st) {
   auto kern = a.L.sf ? attend_kernel<1> : attend_kernel<0>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  // pairs of 256-query CTAs; an odd count gets one CTA with no queries
-  const unsigned blocks = (unsigned)((a.Nq + 255) / 256);
-  dim3 grid((blocks + 1) & ~1u, (unsigned)a.L.H);
-  kern<<<grid, NT, SMEM_BYTES, st>>>(a, slots);
+  // one CTA pair per work unit or part
+  const int64_t pairs = (int64_t)a.n_whole + (int64_t)(a.n_units - a.n_whole) * a.nparts;
+  kern<<<dim3((unsigned)(2 * pairs)), NT, SMEM_BYTES, st>>>(a, slots);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || a.n_units == a.n_whole) return e;
+  const int64_t warps = (int64_t)(a.n_units - a.n_whole) * 512;
+  attend_combine<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 

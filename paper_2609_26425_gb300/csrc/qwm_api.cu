@@ -304,8 +304,18 @@ qwm_status qwm_quantize_append_full(const qwm_config* cfg, qwm_cache* c, const v
   return quantize_append(cfg, c, k, v, N, k_centroids, v_centroids, w, U, Mq, stream);
 }
 
-qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, int64_t Nq, const void* k_cur,
-                      const void* v_cur, int64_t N_cur, float sm_scale, void* out, float* lse, void* stream) {
+namespace {
+
+int device_sms() {
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return nsm;
+}
+
+qwm_status attend_impl(const qwm_config* cfg, const qwm_cache* c, const void* q, int64_t Nq, const void* k_cur,
+                       const void* v_cur, int64_t N_cur, float sm_scale, void* out, float* lse, void* workspace,
+                       size_t workspace_bytes, void* stream) {
   if (!cfg || !c || Nq < 0 || N_cur < 0) return QWM_ERR_INVALID_ARG;
   if (!supported(cfg)) return QWM_ERR_UNSUPPORTED;
   if (!same_shape(cfg, &c->cfg)) return QWM_ERR_INVALID_ARG;
@@ -314,6 +324,7 @@ qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, 
   if (!q || !out) return QWM_ERR_INVALID_ARG;
   if (N_cur > 0 && (!k_cur || !v_cur || !aligned16(k_cur) || !aligned16(v_cur))) return QWM_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out)) return QWM_ERR_INVALID_ARG;
+  if (workspace && (reinterpret_cast<uintptr_t>(workspace) & 255u)) return QWM_ERR_INVALID_ARG;
   if (!(sm_scale > 0.0f) || sm_scale > 3.0e38f) return QWM_ERR_INVALID_ARG;
   if (Nq > ((int64_t)1 << 31) || N_cur > ((int64_t)1 << 31)) return QWM_ERR_UNSUPPORTED;
   int32_t n = qwm_cache_num_chunks(c);
@@ -341,7 +352,41 @@ qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, 
   a.lse = lse;
   a.wait_ns = c->wait_ns;
   a.idle_role = c->idle_role;
+  const int nsm = device_sms();
+  if (nsm <= 0) return QWM_ERR_CUDA;
+  qwm::AttendPlan pl = qwm::plan_attend(Nq, c->L.H, n + (N_cur > 0 ? 1 : 0), nsm, workspace != nullptr);
+  const size_t need = qwm::attend_workspace_bytes(pl);
+  if (need > 0 && workspace_bytes < need) pl = qwm::plan_attend(Nq, c->L.H, n + (N_cur > 0 ? 1 : 0), nsm, false);
+  a.bph = pl.bph;
+  a.n_units = pl.n_units;
+  a.n_whole = pl.n_whole;
+  a.nparts = pl.nparts;
+  if (pl.nparts > 1) {
+    a.part_o = static_cast<float*>(workspace);
+    a.part_ml = a.part_o + (size_t)(pl.n_units - pl.n_whole) * pl.nparts * 512 * 128;
+  }
   return qwm::launch_attend(a, slots, static_cast<cudaStream_t>(stream)) == cudaSuccess ? QWM_OK : QWM_ERR_CUDA;
+}
+
+}  // namespace
+
+qwm_status qwm_attend(const qwm_config* cfg, const qwm_cache* c, const void* q, int64_t Nq, const void* k_cur,
+                      const void* v_cur, int64_t N_cur, float sm_scale, void* out, float* lse, void* stream) {
+  return attend_impl(cfg, c, q, Nq, k_cur, v_cur, N_cur, sm_scale, out, lse, nullptr, 0, stream);
+}
+
+size_t qwm_attend_workspace_bytes(const qwm_config* cfg, const qwm_cache* c, int64_t Nq, int64_t N_cur) {
+  if (!cfg || !c || Nq < 1 || N_cur < 0 || !supported(cfg) || !same_shape(cfg, &c->cfg)) return 0;
+  const int nsm = device_sms();
+  if (nsm <= 0) return 0;
+  const int n_key_units = qwm_cache_num_chunks(c) + (N_cur > 0 ? 1 : 0);
+  return qwm::attend_workspace_bytes(qwm::plan_attend(Nq, c->L.H, n_key_units, nsm, true));
+}
+
+qwm_status qwm_attend_ws(const qwm_config* cfg, const qwm_cache* c, const void* q, int64_t Nq, const void* k_cur,
+                         const void* v_cur, int64_t N_cur, float sm_scale, void* out, float* lse, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  return attend_impl(cfg, c, q, Nq, k_cur, v_cur, N_cur, sm_scale, out, lse, workspace, workspace_bytes, stream);
 }
 
 qwm_status qwm_cache_set_wait_limit(qwm_cache* c, uint64_t ns) {

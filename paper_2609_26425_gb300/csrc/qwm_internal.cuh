@@ -156,7 +156,21 @@ struct AttendArgs {
   float* lse;                  // [H][Nq] or null
   uint64_t wait_ns;            // limit of every bounded wait
   int32_t idle_role;           // QWM_ROLE_*: a role that publishes nothing (test hook), 0 = none
+  // work units (CTA pairs of 512 queries of one head) and their split: units
+  // [0, n_whole) run over every key; each later unit runs as nparts parts over
+  // contiguous ranges of the key units, combined by a second kernel from the
+  // parts' unnormalised O rows and running (max, sum) in part_o / part_ml
+  int32_t bph, n_units, n_whole, nparts;
+  float* part_o;               // [tail units][nparts][512][128] fp32
+  float* part_ml;              // [tail units][nparts][512][2] fp32
 };
+struct AttendPlan {
+  int32_t bph, n_units, n_whole, nparts;
+};
+// The split of a launch: whole units in full waves of the SMs' CTA pairs, the
+// remaining units in parts over the key units (split = false: no parts).
+AttendPlan plan_attend(int64_t Nq, int H, int n_key_units, int nsm, bool split);
+size_t attend_workspace_bytes(const AttendPlan& pl);
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t s);
 
 struct FitArgs {

@@ -114,7 +114,10 @@ def run_workload(wl, *, layer=0, appended=None, r=None, n_tok=96, heads=(0, 1), 
 
     # the new chunk: its queries attend the cache plus its own bf16 K/V (the active chunk)
     q, k, v = src.chunk(appended)
-    out, lse = qwm.qwm_attend(cfg, hist, dev(q), dev(k), dev(v), want_lse=True)
+    # in the launch configuration the bench times: the work units of the
+    # last wave split along the key chunks (qwm_attend_ws)
+    ws = qwm.attend_workspace(cfg, hist, q.shape[0], k.shape[0])
+    out, lse = qwm.qwm_attend(cfg, hist, dev(q), dev(k), dev(v), want_lse=True, workspace=ws)
     torch.cuda.synchronize()
     assert hist.status() == 0
     Ks, Vs = [], []
@@ -192,8 +195,9 @@ def test_microbench_sweep_extremes(H, chunks, C, G, r, Nq, Ncur):
     q = synth.gaussian_bf16(9500 + C, Nq, H, 128)
     kcur = synth.gaussian_bf16(9501 + C, Ncur, H, 128) if Ncur else None
     vcur = synth.gaussian_bf16(9502 + C, Ncur, H, 128) if Ncur else None
+    ws = qwm.attend_workspace(cfg, cache, Nq, Ncur)
     out, lse = qwm.qwm_attend(cfg, cache, dev(q), None if kcur is None else dev(kcur),
-                              None if vcur is None else dev(vcur), want_lse=True)
+                              None if vcur is None else dev(vcur), want_lse=True, workspace=ws)
     torch.cuda.synchronize()
     assert cache.status() == 0
     if Ncur:

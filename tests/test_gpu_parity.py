@@ -319,18 +319,26 @@ def build_cache_and_reference(H, chunk_sizes, C, G, r, M, seed, *, Ncur, Nq, win
     return cfg, cache, q, kcur, vcur, ref, lse
 
 
+@pytest.mark.parametrize("split", [False, True])
 @pytest.mark.parametrize("H,chunks,C,G,r,Ncur,Nq", [
     (4, [880, 880], 64, 32, 16, 880, 880),    # the single-layer workload
     (2, [300, 77], 16, 64, 8, 129, 200),
     (2, [256, 256], 256, 32, 32, 0, 130),     # no active chunk
     (2, [128], 64, 32, 0, 1, 1),              # r = 0, one query, one active key
     (1, [1, 5], 4, 32, 16, 0, 33),            # tiny chunks
+    (3, [300, 200, 129, 77], 16, 32, 16, 50, 1100),  # four chunks and an active one, ragged query blocks
 ])
-def test_attend_parity(H, chunks, C, G, r, Ncur, Nq):
+def test_attend_parity(H, chunks, C, G, r, Ncur, Nq, split):
+    """Attention against the oracle's fp64 softmax; split: through
+    qwm_attend_ws, whose work units are split along the key chunks (every unit
+    here: they are fewer than the GPU's CTA pairs) and combined."""
     cfg, cache, q, kc, vc, ref, lse = build_cache_and_reference(H, chunks, C, G, r, 4, seed=31 * H + Nq,
                                                                Ncur=Ncur, Nq=Nq)
+    ws = qwm.attend_workspace(cfg, cache, Nq, Ncur) if split else None
+    if split:
+        assert ws is not None and ws.numel() > 0  # more than one key unit: the parts are used
     out, lse_g = qwm.qwm_attend(cfg, cache, dev(q), dev(kc) if Ncur else None, dev(vc) if Ncur else None,
-                                want_lse=True)
+                                want_lse=True, workspace=ws)
     torch.cuda.synchronize()
     assert cache.status() == 0
     compare_attention(out.float().cpu().numpy(), ref)
