@@ -445,7 +445,7 @@ __global__ void __launch_bounds__(XNT, 1)
       if (!all_cand) {
         uint8_t* myl = rowbuf;
         constexpr int kList = 16;
-        const int nchunk = (Npad + 31) >> 5;  // 32-column blocks (at most 256 columns)
+        const int npair = (Npad + 63) >> 6;  // pairs of 32-column blocks (at most 256 columns)
         // dt of 32 consecutive columns from their D values, two at a time with
         // packed fused multiply-adds (each lane rounds once, as fmaf(-2, D, A))
         auto dt32 = [&](int cb, float (&v)[32]) {
@@ -464,13 +464,14 @@ __global__ void __launch_bounds__(XNT, 1)
 #pragma unroll
         for (int i = 0; i < 16; ++i) gm[i] = INFINITY;
 #pragma unroll 1
-        for (int cb = 0; cb < nchunk; ++cb) {
-          float va[32];
+        for (int cp = 0; cp < npair; ++cp) {
+          float va[32], vb[32];
           __syncwarp();
-          tmem_ld32(tD + lrow + cb * 32, va);
-          dt32(cb, va);
+          tmem_ld32x2(tD + lrow + cp * 64, tD + lrow + cp * 64 + 32, va, vb);
+          dt32(2 * cp, va);
+          dt32(2 * cp + 1, vb);
 #pragma unroll
-          for (int e = 0; e < 16; ++e) gm[e] = fmin3(gm[e], va[e], va[e + 16]);
+          for (int e = 0; e < 16; ++e) gm[e] = fmin3(fmin3(gm[e], va[e], va[e + 16]), vb[e], vb[e + 16]);
         }
         float tq[CAPT];
 #pragma unroll
@@ -483,6 +484,15 @@ __global__ void __launch_bounds__(XNT, 1)
           tq[0] = fminf(tq[0], x);
         }
         const float T = sel_at(tq, Mc);
+        // The band of step c (every j with dt_j <= kth + 2 B) lies at or below
+        // T2 = T + 2 Bmax: kth (the M-th smallest dt) is at most T and at least
+        // the smallest dt, tq[0], so the bound B below is at most Bmax.  The
+        // second pass lists every column at or below T2, which holds the M + 1
+        // smallest and the whole band.
+        const float an = sqrtf(an2) * 1.0001f;
+        const float Bmax = ldexpf(an * Mn, -13) * 1.25f +
+                           ldexpf(Am + fabsf(K0) + fmaxf(fabsf(tq[0]), fabsf(T)), -16) + 1e-30f;
+        const float T2 = T + 2.0f * Bmax;
 
         float* stash = reinterpret_cast<float*>(rowbuf);
         uint2* lst = reinterpret_cast<uint2*>(rowbuf + 128);
@@ -493,16 +503,20 @@ __global__ void __launch_bounds__(XNT, 1)
         for (int i = 0; i < CAPT; ++i) { tv[i] = INFINITY; tj[i] = 0x7FFFFFFF; }
         int cnt = 0;
 #pragma unroll 1
-        for (int cb = 0; cb < nchunk; ++cb) {
-          float va[32];
+        for (int cp = 0; cp < npair; ++cp) {
+          float va[32], vb[32];
           __syncwarp();
-          tmem_ld32(tD + lrow + cb * 32, va);
-          dt32(cb, va);
-          {
-            const float (&v)[32] = va;
-            uint32_t mk = 0;
+          tmem_ld32x2(tD + lrow + cp * 64, tD + lrow + cp * 64 + 32, va, vb);
+          dt32(2 * cp, va);
+          dt32(2 * cp + 1, vb);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) mk |= (v[e] <= T ? 1u : 0u) << e;
+          for (int hb = 0; hb < 2; ++hb) {
+            const float (&v)[32] = hb ? vb : va;
+            const int cb = 2 * cp + hb;
+            uint32_t m8[4] = {0u, 0u, 0u, 0u};  // four independent partial masks
+#pragma unroll
+            for (int e = 0; e < 32; ++e) m8[e & 3] |= (v[e] <= T2 ? 1u : 0u) << e;
+            uint32_t mk = (m8[0] | m8[1]) | (m8[2] | m8[3]);
             if (mk) {
 #pragma unroll
               for (int k4 = 0; k4 < 8; ++k4)
@@ -530,10 +544,9 @@ __global__ void __launch_bounds__(XNT, 1)
         // fp32 product a = w o k and its bf16 split add 2^-17 |a| |mu_j| (the
         // factor 1.25 holds both); the fp32 A_j and the oracle's sequential
         // sums 2^-17 of their magnitudes each (the 2^-16 term).
-        const float an = sqrtf(an2) * 1.0001f;
         const float Bb = ldexpf(an * Mn, -13) * 1.25f + ldexpf(Am + fabsf(K0) + fabsf(kth), -16) + 1e-30f;
         const float lim = kth + 2.0f * Bb;
-        // a list overflow (more than kList columns at or below T) or a row or
+        // a list overflow (more than kList columns at or below T2) or a row or
         // table that is not finite is left to the exact rescoring of every
         // centroid
         const bool over = cnt > kList || !(an2 < INFINITY) || !(lim < INFINITY);
@@ -545,10 +558,8 @@ __global__ void __launch_bounds__(XNT, 1)
             if (s < Mc) myl[1 + s] = (uint8_t)tj[s < CAPT ? s : 0];
         }
         // The band (every j with dt_j <= kth + 2B, ascending j) of the rows
-        // that are not decided: from the list when it covers the band
-        // (lim <= T), otherwise from all columns.
-        const bool need_band = !over && !decided;
-        if (need_band && lim <= T) {
+        // that are not decided, from the list (lim <= T2)
+        if (!over && !decided) {
           int c2 = 0;
           for (int i = 0; i < mc; ++i) {
             const uint2 en = lst[i];
@@ -558,26 +569,6 @@ __global__ void __launch_bounds__(XNT, 1)
             c2 += take ? 1 : 0;
           }
           n = c2 <= kBand ? c2 : kRecAll;
-        }
-        const bool need_scan = need_band && !(lim <= T);
-        if (__any_sync(0xFFFFFFFFu, need_scan)) {
-          int c2 = 0;
-#pragma unroll 1
-          for (int cb = 0; cb < nchunk; ++cb) {
-            float va[32];
-            __syncwarp();
-            tmem_ld32(tD + lrow + cb * 32, va);
-            dt32(cb, va);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const float x = va[e];
-              const bool take = need_scan && x <= lim;
-              const int sl = c2 < kBand ? c2 : kBand - 1;
-              if (take) myl[1 + sl] = (uint8_t)(cb * 32 + e);
-              c2 += take ? 1 : 0;
-            }
-          }
-          if (need_scan) n = c2 <= kBand ? c2 : kRecAll;
         }
         myl[0] = (uint8_t)n;
         const uint4 r0 = lds16(myl), r1 = lds16(myl + 16);
