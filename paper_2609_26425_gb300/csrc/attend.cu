@@ -183,29 +183,30 @@ __device__ __forceinline__ void qu_to_smem(uint8_t* sQU, int i, int row, uint32_
 
 // SF: the slot's scale format (0: binary16 group scales; 1: uint8 group codes
 // times a binary16 secondary scale per token, App. D.1).
-template <int SF>
+// PARTS: the launch of the tail units' parts (see plan_attend) instead of
+// the whole units.
+template <int SF, bool PARTS>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     attend_kernel(const AttendArgs a, const AttendSlots S) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const Layout& L = a.L;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  // Grid: x = 2 * (pair index) + rank (the CTA pair of a cluster).  Pair
-  // index P < n_whole is the work unit P = h * (blocks of 512 queries per
-  // head) + block, over every key; the later pairs are the parts of the tail
-  // units, each over a contiguous range of the key units (cached chunks, then
-  // the active chunk), whose partial results a second kernel combines.  The
-  // pairs of one head run close together and share its packed tiles through L2.
+  // Whole units: grid x = 2 * (block of 512 queries) + rank (the CTA pair of
+  // a cluster), y = head, every key (the pairs of one head run close together
+  // and share its packed tiles through L2).  Parts: grid x = 2 * (part index)
+  // + rank over the tail units (the units from n_whole on, nparts parts each,
+  // every part over a contiguous range of the key units: cached chunks, then
+  // the active chunk), whose partial results a third kernel combines.
   const int P = blockIdx.x >> 1;
-  const bool whole = P < a.n_whole;
-  const int wunit = whole ? P : a.n_whole + (P - a.n_whole) / a.nparts;
-  const int part = whole ? 0 : (P - a.n_whole) % a.nparts;
-  const int h = wunit / a.bph;
+  const int wunit = PARTS ? a.n_whole + P / a.nparts : (int)blockIdx.y * a.bph + P;
+  const int part = PARTS ? P % a.nparts : 0;
+  const int h = PARTS ? wunit / a.bph : (int)blockIdx.y;
   const int H = L.H, r = L.r;
   const int rpad = r == 8 ? 16 : r;
   const int gshift = L.G == 32 ? 5 : 6;
   const uint32_t rank = cluster_rank();  // 0: leader
-  const int64_t pair0 = (int64_t)(wunit - h * a.bph) * 512;
+  const int64_t pair0 = PARTS ? (int64_t)(wunit - h * a.bph) * 512 : (int64_t)P * 512;
   const int64_t q0 = pair0 + 256 * rank;
   // Q tiles the pair runs: the second is left out when neither CTA has a
   // query in it (the tail of the query range), halving that pair's MMA and
@@ -213,8 +214,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   const int nqt = pair0 + 128 < a.Nq ? 2 : 1;
   const int n_all = S.n + (a.Ncur > 0 ? 1 : 0);
   // this pair's key units [cu0, cu1)
-  const int cu0 = whole ? 0 : (int)((int64_t)part * n_all / a.nparts);
-  const int cu1 = whole ? n_all : (int)((int64_t)(part + 1) * n_all / a.nparts);
+  const int cu0 = PARTS ? (int)((int64_t)part * n_all / a.nparts) : 0;
+  const int cu1 = PARTS ? (int)((int64_t)(part + 1) * n_all / a.nparts) : n_all;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + OFF_BAR + NBAR * 8);
@@ -410,7 +411,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       if (ok && u + 1 < cu1 && unit_at(a, S, u + 1, h).psac) ok = take_qu();
     }
     if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFINAL), 0, a.wait_ns));
-    if (ok && (int)(blockIdx.x >> 1) < a.n_whole) {  // (recomputed: nothing kept live across the loop)
+    if (ok && !PARTS) {
       tc_fence_after();
       const float inv_l = 1.0f / l_run;
       float v[32];
@@ -432,7 +433,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       // a part of a tail unit: the unnormalised O row, the running maximum and
       // sum, for the combining kernel
       tc_fence_after();
-      const size_t prow = ((size_t)((int)(blockIdx.x >> 1) - a.n_whole) * 512 + 256 * rank + 128 * i + row);
+      const size_t prow = ((size_t)(blockIdx.x >> 1) * 512 + 256 * rank + 128 * i + row);
       float v[32];
 #pragma unroll
       for (int cb = 0; cb < 4; ++cb) {
@@ -450,8 +451,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     // Off the critical path: this CTA's share of the active chunk's rows of
     // head h (the rebuild converts them with saturation) is checked for values
     // beyond the binary16 range, which only the status word reports.
-    const int P2 = (int)(blockIdx.x >> 1);
-    if (a.Ncur > 0 && (P2 < a.n_whole || (P2 - a.n_whole) % a.nparts == 0)) {
+    if (a.Ncur > 0 && (!PARTS || (int)(blockIdx.x >> 1) % a.nparts == 0)) {
       const int64_t gx = 2 * (int64_t)a.bph, bx = 2 * (pair0 >> 9) + rank;
       const int64_t per = (a.Ncur + gx - 1) / gx;
       const int64_t r0 = bx * per, r1 = min(a.Ncur, r0 + per);
@@ -905,7 +905,8 @@ AttendPlan plan_attend(int64_t Nq, int H, int n_key_units, int nsm, bool split) 
   pl.nparts = 1;
   const int slots = nsm / 2 > 0 ? nsm / 2 : 1;
   if (!split || n_key_units < 2 || pl.n_units % slots == 0) return pl;
-  const int whole = pl.n_units / slots * slots, tail = pl.n_units - whole;
+  // whole units: full waves of the pair slots, rounded down to whole heads
+  const int whole = pl.n_units / slots * slots / pl.bph * pl.bph, tail = pl.n_units - whole;
   // parts per tail unit: the fewest rounds of the tail over the pair slots
   // times the largest part (in key units), each part charged a fixed 0.15 of
   // a key unit; ties to fewer parts
@@ -930,14 +931,23 @@ size_t attend_workspace_bytes(const AttendPlan& pl) {
 }
 
 cudaError_t launch_attend(const AttendArgs& a, const AttendSlots& slots, cudaStream_t st) {
-  auto kern = a.L.sf ? attend_kernel<1> : attend_kernel<0>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  auto whole = a.L.sf ? attend_kernel<1, false> : attend_kernel<0, false>;
+  auto parts = a.L.sf ? attend_kernel<1, true> : attend_kernel<0, true>;
+  cudaError_t e = cudaFuncSetAttribute(whole, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(parts, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  // one CTA pair per work unit or part
-  const int64_t pairs = (int64_t)a.n_whole + (int64_t)(a.n_units - a.n_whole) * a.nparts;
-  kern<<<dim3((unsigned)(2 * pairs)), NT, SMEM_BYTES, st>>>(a, slots);
+  // the whole units are whole heads (n_whole a multiple of bph): a CTA pair
+  // per block of 512 queries of each of those heads
+  if (a.n_whole > 0) {
+    whole<<<dim3((unsigned)(2 * a.bph), (unsigned)(a.n_whole / a.bph)), NT, SMEM_BYTES, st>>>(a, slots);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  if (a.n_units == a.n_whole) return cudaSuccess;
+  const int64_t pairs = (int64_t)(a.n_units - a.n_whole) * a.nparts;
+  parts<<<dim3((unsigned)(2 * pairs)), NT, SMEM_BYTES, st>>>(a, slots);
   e = cudaGetLastError();
-  if (e != cudaSuccess || a.n_units == a.n_whole) return e;
+  if (e != cudaSuccess) return e;
   const int64_t warps = (int64_t)(a.n_units - a.n_whole) * 512;
   attend_combine<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(a);
   return cudaGetLastError();
