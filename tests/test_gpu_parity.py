@@ -108,7 +108,7 @@ def test_append_parity_two_level_scales(H, N, C, G, r, M):
 
 
 @pytest.mark.parametrize("H,N,C,r,M,use_U", [
-    (2, 300, 64, 16, 4, True),       # the filter + quantize path, ragged tail tile
+    (2, 300, 64, 16, 4, True),       # the fused kernel's candidate filter, ragged tail tile
     (2, 257, 16, 8, 4, True),        # r = 8: a tile needs two dropped rows to go sparse
     (3, 130, 64, 32, 1, True),
     (2, 200, 8, 16, 8, True),        # exhaustive QSAC (M = C)
