@@ -345,6 +345,28 @@ def test_attend_parity(H, chunks, C, G, r, Ncur, Nq, split):
     assert np.abs(lse_g.cpu().numpy() - lse).max() < 2e-2
 
 
+def test_attend_workspace_sizing_and_small_buffer():
+    """qwm_attend_ws needs no scratch over a single key unit; a buffer smaller
+    than qwm_attend_workspace_bytes runs the unsplit launch (the same bits as
+    qwm_attend); the split launch agrees with the oracle and with the unsplit
+    output within the attention tolerance."""
+    cfg, cache, q, _, _, _, _ = build_cache_and_reference(2, [300], 16, 32, 16, 4, seed=5, Ncur=0, Nq=200)
+    assert qwm.qwm_attend_workspace_bytes(cfg, cache, 200, 0) == 0
+    assert qwm.attend_workspace(cfg, cache, 200, 0) is None
+    cfg, cache, q, kc, vc, ref, _ = build_cache_and_reference(2, [300, 77], 16, 32, 16, 4, seed=6, Ncur=129, Nq=200)
+    need = qwm.qwm_attend_workspace_bytes(cfg, cache, 200, 129)
+    assert need > 0
+    plain = qwm.qwm_attend(cfg, cache, dev(q), dev(kc), dev(vc))
+    small = torch.empty(256, dtype=torch.uint8, device="cuda")
+    fallback = qwm.qwm_attend(cfg, cache, dev(q), dev(kc), dev(vc), workspace=small)
+    split = qwm.qwm_attend(cfg, cache, dev(q), dev(kc), dev(vc), workspace=qwm.attend_workspace(cfg, cache, 200, 129))
+    torch.cuda.synchronize()
+    assert cache.status() == 0
+    assert torch.equal(plain, fallback)
+    compare_attention(split.float().cpu().numpy(), ref)
+    assert (split.float() - plain.float()).abs().max().item() < 2e-2
+
+
 @pytest.mark.parametrize("H,chunks,C,G,r,Ncur,Nq", [
     (4, [880, 880], 64, 32, 16, 880, 880),
     (2, [300, 77], 16, 64, 8, 129, 200),
