@@ -761,18 +761,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     }
     if (!ok) *s_err = 1;
   } else {
-    // ------------------------------------------------------------ MMA issue (leader, one thread)
+    // ------------------------------------------------------------ MMA issue (leader, one warp)
     // Order per KV tile j: P0 V(j), S0(j+1), P1 V(j), S1(j+1), so that the
     // softmax of Q tile 0 on tile j+1 overlaps the softmax of Q tile 1 on
     // tile j (S_i(j+1) reuses the TMEM columns of P_i(j) after P_i V(j) has
-    // read them: MMAs of one thread run in issue order).
-    if (rank == 0 && lane == 0) {
-      const uint32_t aQ = smem_u32(sm + OFF_Q), aQU = smem_u32(sm + OFF_QU);
-      const uint32_t aK = smem_u32(sm + OFF_K), aC = smem_u32(sm + OFF_C), aV = smem_u32(sm + OFF_V);
-      const uint32_t aU = smem_u32(sm + OFF_U);
+    // read them: MMAs of one thread run in issue order).  The whole warp runs
+    // the loop; one elected lane issues every MMA and commit.
+    if (rank == 0) {
+      const uint32_t e = elect_one();
+      // operand descriptors: the base of each buffer once, then byte offsets
+      // >> 4 added to the start-address field (every address stays below the
+      // 256 KB that the 14-bit field covers)
+      const uint64_t dQ = desc_sw128(smem_u32(sm + OFF_Q)), dQU = desc_sw128(smem_u32(sm + OFF_QU));
+      const uint64_t dK = desc_sw128(smem_u32(sm + OFF_K)), dC = desc_sw128(smem_u32(sm + OFF_C));
+      const uint64_t dV = desc_sw128(smem_u32(sm + OFF_V)), dU = desc_sw128(smem_u32(sm + OFF_U));
+      auto off = [](int bytes) { return (uint64_t)(bytes >> 4); };
       constexpr uint32_t idS = idesc_f16(256, 128, false);
       constexpr uint32_t idQU = idesc_f16(256, 64, false);
       constexpr uint32_t idPV = idesc_f16(256, 128, true);
+      auto wait_all = [&](int b, uint32_t ph) -> bool {
+        return __all_sync(0xFFFFFFFFu, mbar_wait_cluster(bar(b), ph, a.wait_ns));
+      };
       int total = 0;
       for (int u = cu0; u < cu1; ++u) total += (unit_at(a, S, u, h).ntok + 127) / 128;
       TileCursor sc;  // next tile to issue S for
@@ -782,9 +791,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       auto issue_S = [&](int i) -> bool {
         const int st = sjt & 1;
         const uint32_t ph = (sjt >> 1) & 1;
-        if (i == 0 && !mbar_wait_cluster(bar(B_KFULL + st), ph, a.wait_ns)) return false;
+        if (i == 0 && !wait_all(B_KFULL + st, ph)) return false;
         if (sc.tl == 0 && sc.u == cu0) {  // Q_i in place
-          if (!mbar_wait_cluster(bar(B_QU + i), qph[i], a.wait_ns)) return false;
+          if (!wait_all(B_QU + i, qph[i])) return false;
           qph[i] ^= 1;
         }
         if (sc.tl == 0 && sc.U.psac) {
@@ -792,15 +801,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           // leader's 32 rows of U_r^T, the follower's zero rows): every MMA
           // that read S_i or Q_i U_r of the previous chunk was issued before.
           tc_fence_after();
-          const uint32_t aUc = aU + (sc.u & 1) * 2 * UBLK;
+          const uint64_t dUc = dU + off((sc.u & 1) * 2 * UBLK);
 #pragma unroll
           for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks)
-              umma2_ss(tbase + 128 * i + 64, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32),
-                       desc_sw128(aUc + kb * UBLK + ks * 32), idQU, (kb | ks) != 0);
-          umma2_commit_both(bar(B_QUMMA + i));
-          if (!mbar_wait_cluster(bar(B_QU + i), qph[i], a.wait_ns)) return false;  // moved into the shared A operand
+              umma2_ss_e(tbase + 128 * i + 64, dQ + off((2 * i + kb) * BLK + ks * 32), dUc + off(kb * UBLK + ks * 32),
+                         idQU, (kb | ks) != 0, e);
+          umma2_commit_both_e(bar(B_QUMMA + i), e);
+          if (!wait_all(B_QU + i, qph[i])) return false;  // moved into the shared A operand
           qph[i] ^= 1;
         }
         tc_fence_after();
@@ -809,14 +818,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
           for (int ks = 0; ks < 4; ++ks)
-            umma2_ss(tS, desc_sw128(aQ + (2 * i + kb) * BLK + ks * 32), desc_sw128(aK + (2 * st + kb) * HBLK + ks * 32),
-                     idS, (kb | ks) != 0);
+            umma2_ss_e(tS, dQ + off((2 * i + kb) * BLK + ks * 32), dK + off((2 * st + kb) * HBLK + ks * 32), idS,
+                       (kb | ks) != 0, e);
         if (sc.U.psac)
           for (int ks = 0; ks < rpad / 16; ++ks)
-            umma2_ss(tS, desc_sw128(aQU + i * rpad * 2 + ks * 32), desc_sw128(aC + st * rpad * 2 + ks * 32), idS, 1u);
-        umma2_commit_both(bar(B_SFULL + i));
+            umma2_ss_e(tS, dQU + off(i * rpad * 2 + ks * 32), dC + off(st * rpad * 2 + ks * 32), idS, 1u, e);
+        umma2_commit_both_e(bar(B_SFULL + i), e);
         if (i == nqt - 1) {
-          umma2_commit_both(bar(B_KEMPTY + st));
+          umma2_commit_both_e(bar(B_KEMPTY + st), e);
           sc.next(a, S, h);
           ++sjt;
         }
@@ -826,20 +835,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       for (int jt = 0; jt < total && ok; ++jt) {
         const int st = jt & 1;
         const uint32_t ph = (jt >> 1) & 1;
-        if (!(ok = mbar_wait_cluster(bar(B_VFULL + st), ph, a.wait_ns))) break;
+        if (!(ok = wait_all(B_VFULL + st, ph))) break;
 #pragma unroll
         for (int i = 0; i < nqt; ++i) {
-          if (!(ok = mbar_wait_cluster(bar(B_PFULL + i), jt & 1, a.wait_ns))) break;
+          if (!(ok = wait_all(B_PFULL + i, jt & 1))) break;
           tc_fence_after();
           const uint32_t tP = tbase + 128 * i, tO = tbase + 256 + 128 * i;
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks)
-            umma2_ts(tO, tP + 8 * ks, desc_sw128(aV + st * BLK + ks * 2048), idPV, (jt > 0 || ks > 0) ? 1u : 0u);
-          if (i == nqt - 1) umma2_commit_both(bar(B_VEMPTY + st));
+            umma2_ts_e(tO, tP + 8 * ks, dV + off(st * BLK + ks * 2048), idPV, (jt > 0 || ks > 0) ? 1u : 0u, e);
+          if (i == nqt - 1) umma2_commit_both_e(bar(B_VEMPTY + st), e);
           if (jt + 1 < total && !(ok = issue_S(i))) break;
         }
       }
-      umma2_commit_both(bar(B_OFINAL));
+      umma2_commit_both_e(bar(B_OFINAL), e);
       if (!ok) {
         // a wait ran out: let the MMAs already issued finish before the
         // pair's TMEM is released

@@ -563,5 +563,50 @@ __device__ __forceinline__ void umma2_commit_both(uint32_t bar) {
       : "memory");
 }
 
+// Warp-wide issue: every lane of the warp runs the issue loop in uniform
+// control flow and the MMAs and commits are predicated on one elected lane.
+// A tcgen05.mma issued from a one-lane branch waits for issue cycles behind
+// the other busy warps of its SM sub-partition (its rate halves with one
+// always-ready neighbour); issued this way it keeps the tensor pipe's rate.
+// Whole warp; returns 1 in exactly one lane.
+__device__ __forceinline__ uint32_t elect_one() {
+  uint32_t e;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "elect.sync _|p, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(e));
+  return e;
+}
+// umma2_ss / umma2_ts / umma2_commit_both, issued only where `e` is nonzero.
+__device__ __forceinline__ void umma2_ss_e(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate, uint32_t e) {
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "@q tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(e)
+      : "memory");
+}
+__device__ __forceinline__ void umma2_ts_e(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate, uint32_t e) {
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "@q tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(e)
+      : "memory");
+}
+__device__ __forceinline__ void umma2_commit_both_e(uint32_t bar, uint32_t e) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\t"
+      "setp.ne.b32 q, %1, 0;\n\t"
+      "@q tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %2;\n\t}" ::"r"(bar),
+      "r"(e), "h"((unsigned short)3)
+      : "memory");
+}
+
 }  // namespace ptx
 }  // namespace qwm
