@@ -238,14 +238,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
   // role in all four warps together, and one lane arrives for all of them
   // with a cluster-scope release (which stalls its warp for hundreds of
   // cycles, so the other three do not pay it).  Returns the common flag.
-  auto handoff = [&](int b, int nb, bool okw) -> bool {
+  // `tmem`: the stage is tensor memory the warps wrote with tcgen05.st (P_i),
+  // waited for and fenced before the hand-off, so the follower's arrival
+  // needs no release of its other memory accesses.
+  auto handoff = [&](int b, int nb, bool okw, bool tmem) -> bool {
     if (rank == 0) {
       __syncwarp();
       if (okw && lane == 0) mbar_arrive(bar(b));
       return okw;
     }
     const bool all = named_bar_and(nb, 128, okw);
-    if (all && (warp & 3) == 0 && lane == 0) mbar_arrive_cluster(mapa(bar(b), 0));
+    if (all && (warp & 3) == 0 && lane == 0) {
+      if (tmem) mbar_arrive_cluster_relaxed(mapa(bar(b), 0));
+      else mbar_arrive_cluster(mapa(bar(b), 0));
+    }
     return all;
   };
 
@@ -405,7 +411,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           l_run += lsum;
           tc_fence_before();
         }
-        ok = handoff(B_PFULL + i, 1 + i, okw);
+        ok = handoff(B_PFULL + i, 1 + i, okw, true);
         if (!ok) break;
       }
       if (ok && u + 1 < cu1 && unit_at(a, S, u + 1, h).psac) ok = take_qu();
@@ -648,7 +654,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
         fence_proxy_async_smem();
       }
-      if (!(ok = handoff(B_KFULL + st, 3, okw))) break;
+      if (!(ok = handoff(B_KFULL + st, 3, okw, false))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
@@ -752,7 +758,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
         fence_proxy_async_smem();
       }
-      if (!(ok = handoff(B_VFULL + st, 4, okw))) break;
+      if (!(ok = handoff(B_VFULL + st, 4, okw, false))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);

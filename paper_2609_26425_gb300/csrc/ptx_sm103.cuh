@@ -503,6 +503,17 @@ __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t cluster_addr) {
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
+// Arrive (relaxed, cluster scope) on an mbarrier given by its cluster address:
+// for a hand-off whose payload is tensor memory written by tcgen05.st, made
+// complete by tcgen05.wait::st and ordered before the arrive by
+// tcgen05.fence::before_thread_sync.  The consumer's acquire wait and
+// tcgen05.fence::after_thread_sync order its MMAs after the arrive.  A release
+// at cluster scope would add nothing for that payload and waits for every
+// memory access the SM has in flight (about 1 K cycles while other warps
+// stream global loads, against about 30 for this form).
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
 // Bounded wait with acquire at cluster scope (arrivals from the peer CTA).
 __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, uint64_t limit_ns = 2000000000ull) {
   auto poll = [&]() -> bool {
