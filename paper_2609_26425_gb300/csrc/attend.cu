@@ -23,8 +23,9 @@
 //                    its U_r^T as the B operand of the Q U_r MMA;
 //   warps 12-15      rebuild this CTA's 64 channels of V_hat (same
 //                    reconstruction, no PSAC) for all 128 keys;
-//   warp 16          allocates the pair's TMEM; in the leader, one thread
-//                    issues every MMA: Q_i U_r once per chunk,
+//   warp 16          allocates the pair's TMEM; in the leader it runs the
+//                    issue loop and one elected lane issues every MMA:
+//                    Q_i U_r once per chunk,
 //                    S_i = [Q_i | Q_i U_r] [K_hat0 | C_hat]^T
 //                    (the PSAC logit term rides along as extra reduction
 //                    columns) and O_i += P_i V_hat with P_i read straight from
@@ -231,7 +232,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       else mbar_arrive_cluster(mapa(bar(i), 0));
     }
   };
-  // Hand-off of a finished stage (KV tile or P_i) to the leader's MMA thread.
+  // Hand-off of a finished stage (KV tile or P_i) to the leader's MMA warp.
   // In the leader each warp arrives on its own barrier b (a CTA-scope
   // release).  In the follower the role's four warps meet at named barrier
   // nb, which also ANDs their `ok` flags so that a timed-out wait ends the
@@ -297,7 +298,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     if (qbad) *s_bad = 1;
     fence_proxy_async_smem();
     arrive_leader(B_QU + i);  // Q_i is in place
-    // Q_i U_r of each chunk that carries PSAC columns: the MMA thread computes
+    // Q_i U_r of each chunk that carries PSAC columns: the MMA warp computes
     // it into columns 64.. of S_i (free while S_i is not in use); this group
     // moves it into the shared A operand of the extra reduction columns.
     if (i < nqt) {
