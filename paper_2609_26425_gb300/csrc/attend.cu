@@ -51,7 +51,7 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kWarps = 17;
+constexpr int kWarps = 18;
 constexpr int NT = kWarps * 32;
 constexpr int W_DQV = 12, W_MMA = 16;
 constexpr float kTauLog2 = 8.0f;
@@ -65,8 +65,10 @@ constexpr int OFF_V = OFF_C + HBLK;      // this CTA's 64 channels of V_hat (128
 constexpr int OFF_U = OFF_V + 2 * BLK;    // U_r^T operand of the Q U_r MMA: chunk parity p, block kb at (2p + kb) * 4 KB
 constexpr int UBLK = 4096;                 // 32 rows x 128 bytes
 constexpr int OFF_BAR = OFF_U + 4 * UBLK;
+// B_KRDY / B_VRDY: the follower's rebuilt stages, relayed to the leader's
+// B_KFULL / B_VFULL by the follower's warps 16 and 17.
 enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_PFULL = 10, B_QU = 12, B_OFINAL = 14,
-       B_QUMMA = 15, NBAR = 17 };
+       B_QUMMA = 15, B_KRDY = 17, B_VRDY = 19, NBAR = 21 };
 static_assert(NBAR * 8 + 16 <= 256, "barrier area");
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;  // + alignment slack
 
@@ -256,6 +258,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     return all;
   };
 
+  // Hand-off of a rebuilt K/V stage: each warp arrives at CTA scope, in the
+  // leader on the leader's barrier b, in the follower on the local barrier
+  // rb that the follower's relay warp forwards to b (so the rebuild warps
+  // never wait for a cluster-scope release).
+  auto stage_done = [&](int b, int rb, bool okw) -> bool {
+    __syncwarp();
+    if (okw && lane == 0) mbar_arrive(bar(rank == 0 ? b : rb));
+    return okw;
+  };
+
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
       mbar_init(bar(B_KFULL + s), 5);    // 4 leader rebuild warps + 1 follower arrival
@@ -265,6 +277,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       mbar_init(bar(B_SFULL + s), 1);
       mbar_init(bar(B_PFULL + s), 5);    // 4 leader softmax warps + 1 follower arrival
       mbar_init(bar(B_QU + s), 8);
+      mbar_init(bar(B_KRDY + s), 4);     // the follower's four K rebuild warps
+      mbar_init(bar(B_VRDY + s), 4);
     }
     mbar_init(bar(B_OFINAL), 1);
     mbar_init(bar(B_QUMMA), 1);         // Q_i U_r MMA commit, both CTAs
@@ -655,7 +669,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
         fence_proxy_async_smem();
       }
-      if (!(ok = handoff(B_KFULL + st, 3, okw, false))) break;
+      if (!(ok = stage_done(B_KFULL + st, B_KRDY + st, okw))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
@@ -759,7 +773,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         }
         fence_proxy_async_smem();
       }
-      if (!(ok = handoff(B_VFULL + st, 4, okw, false))) break;
+      if (!(ok = stage_done(B_VFULL + st, B_VRDY + st, okw))) break;
       // the next tile's ids and zero-points are fetched only now: a release
       // waits for every memory operation the thread has in flight
       idn = load_ids(nc);
@@ -774,7 +788,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
     // tile j (S_i(j+1) reuses the TMEM columns of P_i(j) after P_i V(j) has
     // read them: MMAs of one thread run in issue order).  The whole warp runs
     // the loop; one elected lane issues every MMA and commit.
-    if (rank == 0) {
+    if (rank == 0 && warp == W_MMA) {
       const uint32_t e = elect_one();
       // operand descriptors: the base of each buffer once, then byte offsets
       // >> 4 added to the start-address field (every address stays below the
@@ -862,6 +876,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
         mbar_wait(bar(B_OFINAL), 0, a.wait_ns);
         *s_err = 1;
       }
+    } else if (rank == 1) {
+      // ---------------------------------------------------------- hand-off relays (follower)
+      // Warp 16 forwards the K stages and warp 17 the V stages: having
+      // acquired the four rebuild warps' CTA-scope arrivals, one lane
+      // arrives on the leader's barrier with a cluster-scope release, which
+      // covers their shared-memory writes and waits for every memory access
+      // the SM has in flight (hundreds to a thousand cycles) in this warp
+      // instead of in the rebuild warps.
+      const bool kside = warp == W_MMA;
+      TileCursor c;
+      c.init(a, S, h, cu0, (!kside && a.idle_role == QWM_ROLE_V_REBUILD) ? cu0 : cu1);
+      bool ok = true;
+      for (uint32_t jt = 0; c.valid() && ok; ++jt, c.next(a, S, h)) {
+        const int st = jt & 1;
+        ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar((kside ? B_KRDY : B_VRDY) + st), (jt >> 1) & 1, a.wait_ns));
+        if (ok && lane == 0) mbar_arrive_cluster(mapa(bar((kside ? B_KFULL : B_VFULL) + st), 0));
+      }
+      if (!ok) *s_err = 1;
     }
     __syncwarp();
   }
