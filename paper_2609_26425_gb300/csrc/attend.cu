@@ -8,7 +8,7 @@
 // operand is split between the CTAs along N, so each CTA rebuilds only half
 // of every 128-key tile -- keys 64c..64c+63 of K_hat0 and C_hat, channels
 // 64c..64c+63 of V_hat for all 128 keys (c = the CTA's rank) -- while each
-// SM still runs its full share of tensor work.  17 warps per CTA with fixed
+// SM still runs its full share of tensor work.  18 warps per CTA with fixed
 // roles that hand work to each other through mbarriers:
 //   warps 0-3, 4-7   softmax of Q tile 0 / 1: thread = query row; reads its
 //                    logit row S_i from TMEM, keeps the running max and sum,
@@ -29,10 +29,11 @@
 //                    S_i = [Q_i | Q_i U_r] [K_hat0 | C_hat]^T
 //                    (the PSAC logit term rides along as extra reduction
 //                    columns) and O_i += P_i V_hat with P_i read straight from
-//                    TMEM.
+//                    TMEM; in the follower it relays the K stages' hand-offs;
+//   warp 17          in the follower, relays the V stages' hand-offs.
 // Rebuild and softmax warps report to the leader's mbarriers (one arrival per
-// warp, remote for the other CTA); MMA completions are committed to the
-// mbarriers of both CTAs.
+// warp; the follower's softmax warps remotely, its rebuild warps through the
+// relays); MMA completions are committed to the mbarriers of both CTAs.
 // TMEM (512 columns per CTA): S0 | S1 | O0 | O1, 128 fp32 columns each; P_i
 // aliases the first 64 columns of S_i.  MMAs of one thread execute in issue
 // order, so S_i of the next tile never overtakes the P_i V_hat MMA that reads
