@@ -235,27 +235,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
       else mbar_arrive_cluster(mapa(bar(i), 0));
     }
   };
-  // Hand-off of a finished stage (KV tile or P_i) to the leader's MMA warp.
-  // In the leader each warp arrives on its own barrier b (a CTA-scope
-  // release).  In the follower the role's four warps meet at named barrier
-  // nb, which also ANDs their `ok` flags so that a timed-out wait ends the
-  // role in all four warps together, and one lane arrives for all of them
-  // with a cluster-scope release (which stalls its warp for hundreds of
-  // cycles, so the other three do not pay it).  Returns the common flag.
-  // `tmem`: the stage is tensor memory the warps wrote with tcgen05.st (P_i),
-  // waited for and fenced before the hand-off, so the follower's arrival
-  // needs no release of its other memory accesses.
-  auto handoff = [&](int b, int nb, bool okw, bool tmem) -> bool {
+  // Hand-off of P_i (tensor memory the softmax warps wrote with tcgen05.st,
+  // waited for and fenced before the hand-off) to the leader's MMA warp.  In
+  // the leader each warp arrives on barrier b.  In the follower the four
+  // warps meet at named barrier nb, which also ANDs their `ok` flags so that
+  // a timed-out wait ends the role in all four warps together, and one lane
+  // arrives for all of them with a relaxed cluster-scope arrive (the payload
+  // needs no release of other memory accesses).  Returns the common flag.
+  auto handoff = [&](int b, int nb, bool okw) -> bool {
     if (rank == 0) {
       __syncwarp();
       if (okw && lane == 0) mbar_arrive(bar(b));
       return okw;
     }
     const bool all = named_bar_and(nb, 128, okw);
-    if (all && (warp & 3) == 0 && lane == 0) {
-      if (tmem) mbar_arrive_cluster_relaxed(mapa(bar(b), 0));
-      else mbar_arrive_cluster(mapa(bar(b), 0));
-    }
+    if (all && (warp & 3) == 0 && lane == 0) mbar_arrive_cluster_relaxed(mapa(bar(b), 0));
     return all;
   };
 
@@ -427,7 +421,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NT, 1)
           l_run += lsum;
           tc_fence_before();
         }
-        ok = handoff(B_PFULL + i, 1 + i, okw, true);
+        ok = handoff(B_PFULL + i, 1 + i, okw);
         if (!ok) break;
       }
       if (ok && u + 1 < cu1 && unit_at(a, S, u + 1, h).psac) ok = take_qu();
